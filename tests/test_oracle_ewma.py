@@ -1,0 +1,93 @@
+"""Pins for the oracle's R10 (revised PPO-EWMA, Sec. 5.2, Eq. 5, App. B).
+
+The App. B recursion is checked against the Eq. 5 closed form (a different
+expression of the same average); the weights sum to one; the stationary
+update is Table 1's plain EWMA; the center of mass and the W/(W+2) rule are
+checked against numerically summed series; resets are exact.
+"""
+
+import math
+
+import numpy as np
+import pytest
+
+from oracle import (EwmaState, beta_for_window, center_of_mass, ewma_closed_form,
+                    ewma_coefficients, ewma_update)
+
+
+@pytest.mark.parametrize("beta", [0.5, 0.75, 0.99])
+def test_recursion_equals_closed_form(beta):
+    rng = np.random.default_rng(1)
+    thetas = [rng.normal(0, 0.02, size=64) for _ in range(10)]
+    st = EwmaState()
+    tp = np.zeros(64)
+    for t, th in enumerate(thetas):
+        tp, st, _ = ewma_update(tp, th, beta, st)
+        np.testing.assert_allclose(tp, ewma_closed_form(thetas[:t + 1], beta), rtol=1e-13,
+                                   atol=1e-16)
+    assert abs(st.w - sum(beta ** k for k in range(10))) < 1e-12
+
+
+def test_first_step_copies_and_weights_sum_to_one():
+    a, b, reset, st = ewma_coefficients(EwmaState(), 0.9)
+    assert (a, b, reset, st.w) == (0.0, 1.0, False, 1.0)
+    st = EwmaState(w=3.7)
+    for _ in range(20):
+        a, b, _, st = ewma_coefficients(st, 0.8)
+        assert abs(a + b - 1.0) < 1e-15
+
+
+def test_constant_parameters_are_a_fixed_point():
+    th = np.linspace(-1, 1, 33)
+    st = EwmaState(w=5.0)
+    tp = th.copy()
+    for _ in range(5):
+        tp, st, _ = ewma_update(tp, th, 0.93, st)
+    np.testing.assert_allclose(tp, th, rtol=1e-15, atol=1e-16)
+
+
+def test_stationary_limit_is_table1_plain_ewma():
+    # Table 1: theta_prox,t = beta theta_prox,t-1 + (1 - beta) theta_t, which is
+    # the recursion at its fixed point w = 1 / (1 - beta).
+    beta = 0.99
+    a, b, _, st = ewma_coefficients(EwmaState(w=1.0 / (1.0 - beta)), beta)
+    assert abs(b - (1.0 - beta)) < 1e-15 and abs(a - beta) < 1e-15
+    assert abs(st.w - 1.0 / (1.0 - beta)) < 1e-12
+
+
+def test_center_of_mass_series_and_window_rule():
+    for beta in (0.5, 0.75, 0.9, 0.99):
+        k = np.arange(20000)
+        w = beta ** k
+        assert abs(math.fsum(k * w) / math.fsum(w) - center_of_mass(beta)) < 1e-9
+    for W in (1, 2, 3, 6, 10):
+        # the rule places the center of mass at the window midpoint W / 2
+        assert abs(center_of_mass(beta_for_window(W)) - W / 2.0) < 1e-12
+    assert beta_for_window(6) == 0.75
+
+
+def test_reset_is_exact_and_counts():
+    rng = np.random.default_rng(2)
+    th = rng.normal(0, 0.02, size=100).astype(np.float32)
+    tp = th + rng.normal(0, 1e-4, size=100).astype(np.float32)
+    st = EwmaState(w=100.0, streak=0, n_resets=2)
+    new, st2, (a, b, reset) = ewma_update(tp, th, 0.99, st, n_active=80, n_valid=100, tau=0.9)
+    assert reset and np.array_equal(new, th.astype(np.float64))
+    assert (st2.w, st2.streak, st2.n_resets) == (1.0, 0, 3)
+    new, st3, (_, _, reset) = ewma_update(tp, th, 0.99, st, n_active=95, n_valid=100, tau=0.9)
+    assert not reset and st3.streak == 0 and st3.n_resets == 2
+
+
+def test_streak_rule():
+    st = EwmaState(w=4.0)
+    seq = [(50, 100), (99, 100), (50, 100), (50, 100), (10, 0), (50, 100)]
+    resets = []
+    for n_act, n_val in seq:
+        _, _, reset, st = ewma_coefficients(st, 0.75, n_active=n_act, n_valid=n_val,
+                                            tau=0.9, min_streak=2)
+        resets.append((reset, st.streak))
+    # low, high (streak cleared), low, low (second in a row: reset), no tokens
+    # (no evidence, streak kept), low
+    assert resets == [(False, 1), (False, 0), (False, 1), (True, 0), (False, 0), (False, 1)]
+    _, _, reset, _ = ewma_coefficients(EwmaState(w=2.0), 0.75, force_reset=True)
+    assert reset
