@@ -1,0 +1,473 @@
+#!/usr/bin/env python
+"""Benchmark of the decoupled off-policy correction hot path on GB300.
+
+One step = the whole path over one batch: K1 (log pi_old of the sampled tokens
+over the old logits), K0 + K2 (fused decoupled loss forward + dlogits) on the
+current logits, and K3 (PPO-EWMA update of 7.6e9 float32 proximal parameters,
+auto-reset fed by K2's statistics).  Workload: T=65536 tokens packed from 128
+sequences, V=151936, bf16 logits (the agentic batch), seeded synthetic data.
+Inputs (40 GB of logits, 61 GB of EWMA buffers) are far larger than L2, so no
+flush is needed between steps.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Prints one JSON line (rank 0).  Under torchrun every rank runs a replica of
+the workload on its own batch (weak scaling); the only exchange is the
+all-reduce of the loss statistics before the EWMA reset decision.
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "correction-loss tokens/s fwd+bwd at V=151936; HBM GB/s vs peak"
+WORKLOAD = "agentic_bf16_v151936"
+EWMA_BETA = 0.99
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--ewma-n", type=int, default=7_600_000_000)
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-rows", type=int, default=96)
+    ap.add_argument("--cpu-params", type=int, default=1 << 25)
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- helpers
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "of measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "of fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling while the timed region runs."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu_id), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except FileNotFoundError:
+            self.proc = None
+            return
+        t0 = time.time()
+        while time.time() - t0 < 5 and os.path.getsize(self.path) == 0:
+            time.sleep(0.05)
+
+    def stop(self, t_begin, t_end):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait(timeout=10)
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                    rows.append((ts, float(parts[1]), float(parts[2]), parts[3], *parts[4:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        inside = [r for r in rows if t_begin - 1 <= r[0] <= t_end + 1] or rows
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = sorted(r[1] for r in inside)
+        reasons = set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in inside:
+            for name, val in zip(names, r[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[2] for r in inside),
+                "samples": len(inside), "reasons": sorted(reasons)}
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2605_12070_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic():
+    """Per-token / per-element DRAM bytes from the committed ncu summary, if the
+    kernels have not changed since it was captured."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except Exception:
+        return {}
+    return d.get("kernels", {}) if d.get("source_hash") == kernel_source_hash() else {}
+
+
+# ----------------------------------------------------------------- the oracle arm
+
+def oracle_sample_times(batch, rows, n_params, threads):
+    """Times the float64 oracle on `rows` tokens and `n_params` EWMA elements.
+    Inputs are copied to the host before the clock starts."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from oracle.rows import map_row_chunks
+    rows = np.asarray(rows)
+    it = torch.as_tensor(rows, device=batch.z_theta.device)
+    zt = batch.z_theta[it].cpu()
+    zo = batch.z_old[it].cpu()
+    ids = batch.ids.cpu().numpy().astype(np.int64)
+    mask = None if batch.mask is None else batch.mask.cpu().numpy()
+    N = int(mask.sum()) if mask is not None else batch.T
+    lmu = batch.logp_mu.cpu().numpy()[rows]
+    adv = batch.adv.cpu().numpy()[rows]
+    m = None if mask is None else mask[rows]
+    p = oracle.LossParams(**batch.thresholds())
+    g = torch.Generator().manual_seed(0)
+    th = torch.randn(n_params, generator=g).numpy()
+    tp = th + 1e-4 * torch.randn(n_params, generator=g).numpy()
+    pos = {int(r): k for k, r in enumerate(rows)}
+
+    def one(chunk):
+        k = np.array([pos[int(r)] for r in chunk])
+        z_old = zo[k].to(torch.float64).numpy()
+        z = zt[k].to(torch.float64).numpy()
+        lo, _ = oracle.token_logprob(z_old, ids[chunk])
+        lt, lse = oracle.token_logprob(z, ids[chunk])
+        terms = oracle.token_terms(lt, lo.astype(np.float32), lmu[k], adv[k],
+                                   None if m is None else m[k], p,
+                                   id_ok=(ids[chunk] >= 0), N=N)
+        dz = oracle.softmax_grad_rows(z, ids[chunk], lse, terms["g"])
+        return float(terms["loss_sum"]) + float(dz[0, 0])
+
+    t0 = time.perf_counter()
+    map_row_chunks(one, rows, chunk=max(1, len(rows) // threads), threads=threads)
+    t_rows = time.perf_counter() - t0
+
+    def ewma_part(ix):
+        sl = slice(int(ix[0]), int(ix[-1]) + 1)
+        oracle.ewma_update(tp[sl], th[sl], EWMA_BETA, oracle.EwmaState(w=1 / (1 - EWMA_BETA)))
+        return 0
+
+    t0 = time.perf_counter()
+    map_row_chunks(ewma_part, np.arange(n_params), chunk=max(1, n_params // threads),
+                   threads=threads)
+    t_par = time.perf_counter() - t0
+    return t_rows, t_par
+
+
+def cpu_baseline(batch, n_params_full, rows_n, params_n):
+    import numpy as np
+
+    from oracle.rows import host_cores
+    threads = host_cores()
+    rng = np.random.default_rng(0)
+    valid = np.nonzero(batch.mask.cpu().numpy())[0] if batch.mask is not None else np.arange(batch.T)
+    rows = np.sort(rng.choice(valid, size=min(rows_n, valid.size), replace=False))
+    t_rows, t_par = oracle_sample_times(batch, rows, params_n, threads)
+    step_s = batch.T * t_rows / rows.size + n_params_full * t_par / params_n
+    return {
+        "value": batch.T / step_s, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+        "sample": (f"float64 numpy oracle on {rows.size} valid tokens of the T={batch.T}, "
+                   f"V={batch.V} batch ({t_rows:.2f} s) and {params_n} EWMA elements "
+                   f"({t_par:.2f} s), scaled to T tokens + {n_params_full} parameters per step"),
+        "seconds": round(t_rows + t_par, 2),
+    }
+
+
+# ----------------------------------------------------------------- main
+
+def main():
+    args = parse_args()
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference" and rank != 0:
+        return
+    if world > 1 and args.impl == "ours":
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2605_12070_gb300 import dp, occ
+    from paper_2605_12070_gb300.workloads import make_ewma_buffers, make_loss_batch
+
+    batch = make_loss_batch(WORKLOAD, seed=rank, device=dev)
+    T, V = batch.T, batch.V
+    n_valid = int(batch.mask.sum().item())
+
+    if args.impl == "reference":
+        run_reference(args, batch, world)
+        return
+
+    theta, theta_prox = make_ewma_buffers(args.ewma_n, seed=rank, device=dev)
+    state = occ.new_ewma_state(dev, w0=1.0 / (1.0 - EWMA_BETA))
+    lp_old = torch.empty(T, dtype=torch.float32, device=dev)
+    dlogits = torch.empty((T, V), dtype=torch.bfloat16, device=dev)
+    logp = torch.empty(T, dtype=torch.float32, device=dev)
+    flags = torch.empty(T, dtype=torch.uint8, device=dev)
+    stats = occ.new_loss_stats(dev)
+    ws = occ.new_workspace(T, V, dev)
+    denom = dp.global_token_count(n_valid) if world > 1 else 0
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        occ.occ_token_logprob(batch.z_old, batch.ids, logp_out=lp_old)
+        if ev is not None:
+            ev[1].record(stream)
+        occ.occ_decoupled_loss_fwd_bwd(batch.z_theta, batch.ids, lp_old, batch.logp_mu, batch.adv,
+                                       batch.mask, **batch.thresholds(), denom=denom,
+                                       dlogits=dlogits, logp_out=logp, flags_out=flags,
+                                       stats=stats, workspace=ws)
+        if world > 1:
+            dp.allreduce_loss_stats(stats)
+        if ev is not None:
+            ev[2].record(stream)
+        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=0.9)
+        if ev is not None:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+    gpu_id = 0
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid).replace("GPU-", "")
+    except Exception:
+        gpu_id = local
+    clocks = ClockSampler(gpu_id)
+    clocks.start()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    t_begin = time.time()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for k in range(args.steps):
+        step(evs[k])
+    end.record(stream)
+    torch.cuda.synchronize()
+    t_end = time.time()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop(t_begin, t_end)
+    elapsed = start.elapsed_time(end) / 1e3
+    if world > 1:
+        t = torch.tensor([elapsed], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    k1 = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps / 1e3
+    k2 = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps / 1e3
+    k3 = sum(e[2].elapsed_time(e[3]) for e in evs) / args.steps / 1e3
+    ms_step = elapsed / args.steps * 1e3
+
+    peak, peak_kind = measured_peak()
+    traffic = ncu_traffic()
+    bytes_k1 = T * V * 2 + T * 8
+    bytes_k2 = n_valid * V * 2 + T * V * 2 + T * 37
+    bytes_k3 = args.ewma_n * 12
+    kern = {
+        "k1_token_logprob": (k1, bytes_k1, T),
+        "k2_decoupled_loss_fwd_bwd": (k2, bytes_k2, T),
+        "k3_ewma_update": (k3, bytes_k3, args.ewma_n),
+    }
+    roof = {}
+    for name, (sec, byts, units) in kern.items():
+        tr = traffic.get(name)
+        achieved = byts / sec / 1e9
+        roof[name] = {
+            "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+            "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+            "traffic": None if tr is None else round(tr["bytes_per_unit"] * units),
+            "algorithmic_bytes": byts, "ms": round(sec * 1e3, 4),
+        }
+    dominant = max(roof, key=lambda k: roof[k]["ms"])
+    loss_ms = (k1 + k2) * 1e3
+    line = {
+        "metric": METRIC,
+        "value": round(world * T / (elapsed / args.steps), 1),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {
+            "workload": (f"decoupled-loss step on T={T} tokens (128 packed sequences, "
+                         f"{n_valid} valid), V={V} bf16 logits (K1 old log-probs + K0/K2 fused "
+                         f"loss fwd+bwd) chained with the PPO-EWMA update of "
+                         f"{args.ewma_n} fp32 parameters (K3)"),
+            "T": T, "V": V, "ewma_params": args.ewma_n, "logits_dtype": "bf16",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": "inputs larger than L2 (40 GB logits, 61 GB EWMA buffers): no flush",
+        },
+        "roofline": dict(roof[dominant], kernel=dominant),
+        "kernels": roof,
+        "loss_only": {"tokens_per_s": round(world * T / ((k1 + k2)), 1), "ms": round(loss_ms, 4),
+                      "hbm_frac": round((bytes_k1 + bytes_k2) / (k1 + k2) / 1e9 / peak, 4)},
+        "gpu_launches": args.steps * 6,
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(batch, args.ewma_n, args.cpu_rows, args.cpu_params)
+    if not args.no_e2e:
+        line["e2e"] = run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits,
+                              logp, flags, denom, world, dev)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _host_available_bytes():
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits, logp, flags, denom,
+            world, dev):
+    """Same step through the public API with the inputs in pinned HOST memory:
+    every step copies the logits, token arrays and the new actor parameters to
+    the device and reads the loss statistics back."""
+    import torch
+
+    from paper_2605_12070_gb300 import dp, occ
+    dev_inputs = [batch.z_old, batch.z_theta, batch.ids, batch.logp_mu, batch.adv, batch.mask,
+                  theta]
+    need = sum(t.numel() * t.element_size() for t in dev_inputs)
+    if _host_available_bytes() < 1.3 * need:
+        return {"value": None, "unit": "tokens/s",
+                "skipped": f"needs {need / 1e9:.0f} GB of pinned host memory, "
+                           f"{_host_available_bytes() / 1e9:.0f} GB available"}
+    host = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in dev_inputs]
+    for h, d in zip(host, dev_inputs):
+        h.copy_(d)
+    stats_h = torch.empty(occ.LOSS_STATS_BYTES, dtype=torch.uint8, pin_memory=True)
+    stream = torch.cuda.current_stream(dev)
+
+    def e2e_step():
+        for h, d in zip(host, dev_inputs):
+            d.copy_(h, non_blocking=True)
+        occ.occ_token_logprob(batch.z_old, batch.ids, logp_out=lp_old)
+        occ.occ_decoupled_loss_fwd_bwd(batch.z_theta, batch.ids, lp_old, batch.logp_mu, batch.adv,
+                                       batch.mask, **batch.thresholds(), denom=denom,
+                                       dlogits=dlogits, logp_out=logp, flags_out=flags,
+                                       stats=stats, workspace=ws)
+        if world > 1:
+            dp.allreduce_loss_stats(stats)
+        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=0.9)
+        stats_h.copy_(stats, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e.record(stream)
+    torch.cuda.synchronize()
+    sec = s.elapsed_time(e) / 1e3 / args.e2e_steps
+    if world > 1:
+        t = torch.tensor([sec], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        sec = float(t.item())
+    occ.decode_loss_stats(stats_h)
+    return {"value": round(world * batch.T / sec, 1), "unit": "tokens/s",
+            "h2d_bytes_per_step": need, "d2h_bytes_per_step": occ.LOSS_STATS_BYTES,
+            "ms_per_step": round(sec * 1e3, 3), "steps": args.e2e_steps}
+
+
+def run_reference(args, batch, world):
+    """The oracle as the reference arm: each step times the float64 oracle on a
+    bounded sample of the same workload (host cores)."""
+    import numpy as np
+
+    from oracle.rows import host_cores
+    threads = host_cores()
+    rng = np.random.default_rng(1)
+    valid = np.nonzero(batch.mask.cpu().numpy())[0]
+    rows_n, params_n = 32, 1 << 23
+    tot_rows = tot_par = 0.0
+    for k in range(args.warmup + args.steps):
+        rows = np.sort(rng.choice(valid, size=rows_n, replace=False))
+        tr, tp = oracle_sample_times(batch, rows, params_n, threads)
+        if k >= args.warmup:
+            tot_rows += tr
+            tot_par += tp
+    step_s = batch.T * (tot_rows / args.steps) / rows_n + args.ewma_n * (tot_par / args.steps) / params_n
+    value = batch.T / step_s
+    sample = (f"per step: float64 oracle on {rows_n} valid tokens of the T={batch.T}, V={batch.V} "
+              f"batch and {params_n} EWMA elements, scaled to the full step")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(step_s * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"oracle on the same T={batch.T}, V={batch.V} step + "
+                               f"{args.ewma_n}-parameter EWMA update", "T": batch.T, "V": batch.V},
+        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": threads,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

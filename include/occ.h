@@ -1,0 +1,201 @@
+/*
+ * occ.h -- C ABI of the GB300 (sm_103a) library for the decoupled off-policy
+ * correction of "Missing Old Logits in Asynchronous Agentic RL" (arXiv 2605.12070).
+ *
+ * The library computes, on one GPU and with hand-written CUDA kernels:
+ *   - per-token log-probabilities of the sampled tokens under a policy's
+ *     logits (the factors of the ratios of Eq. 1);
+ *   - the decoupled PPO loss: the discrepancy ratio r_d = pi_old / mu_old is
+ *     masked to a band (Eq. 4), the staleness ratio r_s = pi_theta / pi_old
+ *     goes through the advantage-sign-dependent PPO clip (Eqs. 2-3), the loss
+ *     is reduced to a token mean, and the gradient with respect to the logits
+ *     is written in the same pass;
+ *   - the revised PPO-EWMA update of the proximal parameters that stand in
+ *     for missing old logits (Eq. 5, App. B), with the auto-reset of Sec. 5.2.
+ *
+ * Conventions shared by every entry point:
+ *   - Every pointer argument is caller-owned DEVICE memory unless marked
+ *     "host".  The library never allocates or frees memory.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ *     default stream).  A returned OCC_OK means the work was enqueued.
+ *   - Arguments are validated on the host before anything is launched; an
+ *     invalid call returns an error status, launches nothing and records a
+ *     message readable with occ_last_error() (per host thread).
+ *   - Data-dependent problems found on the device (a token id outside
+ *     [0, V)) never trap: the token is dropped and a bit is set in
+ *     occ_loss_stats.err.
+ *   - Logits are row-major [T, V] with a row stride `ld` >= V elements.
+ *     Rows whose start is 16-byte aligned (base address and ld * element size
+ *     multiples of 16) use the vectorised kernels; any other layout runs on a
+ *     scalar-load kernel of the same library, with identical results.
+ */
+#ifndef OCC_H_
+#define OCC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define OCC_VERSION 1
+
+typedef enum {
+  OCC_OK = 0,
+  OCC_ERR_INVALID_ARG = 1, /* null pointer, negative size, ld < V, bad threshold, overlap */
+  OCC_ERR_UNSUPPORTED = 2, /* dtype or size the library does not handle             */
+  OCC_ERR_MISALIGNED = 3,  /* a scalar array not aligned to its element size         */
+  OCC_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed                   */
+  OCC_ERR_WORKSPACE = 5    /* workspace missing or smaller than occ_loss_workspace_bytes */
+} occ_status;
+
+typedef enum { OCC_F32 = 0, OCC_BF16 = 1 } occ_dtype;
+
+/* Bits of occ_loss_stats.err (device-detected data problems). */
+#define OCC_DATA_ERR_BAD_ID 1 /* some token id was outside [0, V); those tokens were dropped */
+
+/* Bits of the per-token flags written by occ_decoupled_loss_fwd_bwd. */
+#define OCC_FLAG_IN_BAND 1 /* r_d inside [rd_lo, rd_hi]                        (Eq. 4) */
+#define OCC_FLAG_CLIPPED 2 /* PPO clip rejects the token, i.e. MIS_ppo = 0      (Eq. 3) */
+#define OCC_FLAG_ACTIVE 4  /* valid, in band and not clipped: carries gradient          */
+#define OCC_FLAG_VALID 8   /* loss mask set and id in range                             */
+
+/* Loss options (HOST struct, read during the call). */
+typedef struct {
+  double rd_lo, rd_hi;      /* inclusive band on r_d, e.g. [1/c, c] (Eq. 4); 0 <= rd_lo <= rd_hi */
+  double eps_low, eps_high; /* clip interval [1 - eps_low, 1 + eps_high] on r_s (Eq. 3, App. A);
+                               0 <= eps_low <= 1, eps_high >= 0                                */
+  double grad_scale;        /* upstream d(objective)/d(loss); multiplies dlogits only (1 = plain) */
+  int64_t denom;            /* > 0: token-mean denominator N given by the caller;
+                               <= 0: N = number of valid tokens, counted on the device        */
+  int32_t rd_weight;        /* 1: token weight M(r_d) r_d (Table 5, "PPO-EWMA & train_infer");
+                               0: weight M(r_d) only (Table 5, "decoupled PPO & train_infer")  */
+  int32_t dlogits_f32;      /* 1: write float32 dlogits even for bf16 logits                   */
+} occ_loss_params;
+
+/* Loss results (DEVICE struct, fully written by every successful call). */
+typedef struct {
+  double loss_sum;   /* sum_t loss_t                                             */
+  double loss;       /* loss_sum / N, 0 when N = 0 (token mean)                  */
+  int64_t n_valid;   /* tokens with mask set and id in range                     */
+  int64_t n_rd_out;  /* valid tokens with r_d outside the band                   */
+  int64_t n_clipped; /* valid tokens rejected by the PPO clip                    */
+  int64_t n_active;  /* valid, in band, not clipped; rho = n_active / n_valid    */
+  int64_t denom;     /* the N that was used                                      */
+  int32_t err;       /* OCC_DATA_ERR_* bits                                      */
+  int32_t reserved;
+} occ_loss_stats;
+
+/* PPO-EWMA state (DEVICE struct, caller-owned; save it with theta_prox to resume). */
+typedef struct {
+  double w;         /* cumulative weight w^(t-1) of App. B: 0 for an empty history,
+                       1/(1-beta) for the stationary (plain EWMA) regime            */
+  double coef_a;    /* coefficients of the last update: theta_prox <- a theta_prox + b theta */
+  double coef_b;
+  int32_t streak;   /* consecutive updates whose rho was below tau               */
+  int32_t n_resets; /* resets performed so far                                   */
+  int32_t last_reset; /* 1 if the last update was a reset                        */
+  int32_t reserved;
+} occ_ewma_state;
+
+/*
+ * occ_token_logprob -- log pi(y_t) for every row of a logits matrix.
+ *
+ * Computes lse[t] = log sum_v exp(logits[t, v]) with a single streaming pass
+ * over the vocabulary, and logp[t] = logits[t, ids[t]] - lse[t].  These are
+ * the per-token factors of the ratios of Eq. 1 (used for pi_old, or for the
+ * proxy pi_prox of Eq. 5 / pi_async of Table 1).
+ *
+ *   logits   [T, ld] row-major, dtype dt (bf16 or f32); only columns [0, V) are read
+ *   T, V, ld T >= 0 rows, V >= 1 columns, row stride ld >= V (elements)
+ *   ids      [T] int32 sampled token ids
+ *   logp_out [T] float32 (written); NaN where ids[t] is outside [0, V)
+ *   lse_out  [T] float32 or NULL
+ * Accumulation is float32 per element with a float64 row epilogue.
+ */
+occ_status occ_token_logprob(const void* logits, occ_dtype dt, int64_t T, int64_t V, int64_t ld,
+                             const int32_t* ids, float* logp_out, float* lse_out, void* stream);
+
+/* Bytes of device workspace occ_decoupled_loss_fwd_bwd needs for T tokens. */
+size_t occ_loss_workspace_bytes(int64_t T, int64_t V);
+
+/*
+ * occ_decoupled_loss_fwd_bwd -- the decoupled PPO loss and its logits gradient.
+ *
+ * For every token t (Sec. 3.2, Eqs. 1-4; Table 5 for the role of r_d):
+ *   m_t      = loss_mask[t] != 0 and 0 <= ids[t] < V  (valid)
+ *   logp_t   = log softmax(logits[t])[ids[t]]
+ *   r_d      = exp(logp_old[t] - logp_mu[t]),   M_d = 1{rd_lo <= r_d <= rd_hi}
+ *   r_s      = exp(logp_t - logp_old[t])
+ *   MIS_ppo  = A_t >= 0 ? r_s <= 1 + eps_high : r_s >= 1 - eps_low
+ *   w_d      = rd_weight ? r_d : 1
+ *   loss_t   = -m_t M_d w_d min(r_s A_t, clip(r_s, 1 - eps_low, 1 + eps_high) A_t)
+ *   loss     = sum_t loss_t / N,  N = sum_t m_t (or params->denom)
+ *   dlogits[t, v] = g_t (1[v = ids[t]] - softmax(logits[t])_v),
+ *   g_t      = -grad_scale m_t M_d MIS_ppo w_d r_s A_t / N
+ * Threshold decisions are taken in log-ratio space in float64.
+ *
+ *   logits     [T, ld] bf16 or f32 (dt); read once
+ *   ids        [T] int32;  logp_old, logp_mu, adv: [T] float32
+ *   loss_mask  [T] uint8 or NULL (= all ones)
+ *   p          HOST pointer to the options
+ *   logp_out   [T] float32 or NULL: logp_t for valid tokens, 0 for dropped ones
+ *   flags_out  [T] uint8 or NULL: OCC_FLAG_* bits (0 for dropped tokens)
+ *   dlogits    [T, ld_grad] or NULL (forward only); dtype = dt, or f32 when
+ *              p->dlogits_f32; may be exactly `logits` (in place, same ld and dtype)
+ *              but must not overlap it otherwise.  Rows of dropped tokens are zero.
+ *   stats      DEVICE occ_loss_stats, fully overwritten
+ *   workspace  DEVICE scratch of at least occ_loss_workspace_bytes(T, V) bytes,
+ *              16-byte aligned; contents need not be initialised
+ * Tokens with m_t = 0 are not read from `logits` at all.  The result is
+ * deterministic (no floating-point atomics).
+ */
+occ_status occ_decoupled_loss_fwd_bwd(const void* logits, occ_dtype dt, int64_t T, int64_t V,
+                                      int64_t ld, const int32_t* ids, const float* logp_old,
+                                      const float* logp_mu, const float* adv,
+                                      const uint8_t* loss_mask, const occ_loss_params* p,
+                                      float* logp_out, uint8_t* flags_out, void* dlogits,
+                                      int64_t ld_grad, occ_loss_stats* stats, void* workspace,
+                                      size_t ws_bytes, void* stream);
+
+/*
+ * occ_ewma_update -- revised PPO-EWMA step on flat float32 parameters.
+ *
+ * App. B recursion: w <- 1 + beta w, theta_prox <- a theta_prox + b theta with
+ * a = beta w_prev / w, b = 1 / w (a + b = 1; the closed form is Eq. 5).
+ * Auto-reset (Sec. 5.2): when `stats` is given and has n_valid > 0, rho =
+ * n_active / n_valid; a step with rho < tau extends `streak`, any other step
+ * clears it; when streak reaches `min_streak` (1 = the paper's rule), or when
+ * force_reset != 0, theta_prox <- theta exactly, w <- 1, streak <- 0.
+ * The decision is taken on the device; the host never waits.
+ *
+ *   theta_prox [n] float32, updated in place;  theta [n] float32
+ *   n          >= 0 elements (64-bit)
+ *   beta       in [0, 1)
+ *   st         DEVICE occ_ewma_state, read and updated
+ *   stats      DEVICE occ_loss_stats of the latest loss step, or NULL (no auto-reset)
+ *   tau        reset threshold on rho;  min_streak >= 1
+ */
+occ_status occ_ewma_update(float* theta_prox, const float* theta, int64_t n, double beta,
+                           occ_ewma_state* st, const occ_loss_stats* stats, double tau,
+                           int32_t min_streak, int32_t force_reset, void* stream);
+
+/* Sets a DEVICE occ_ewma_state to {w = w0, streak = 0, n_resets = 0}: w0 = 0 for an
+ * empty history, 1/(1-beta) to start in the stationary regime. */
+occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* stream);
+
+/* Static description of a status code. */
+const char* occ_status_string(occ_status s);
+
+/* Message of the last failed call on this host thread ("" if none). */
+const char* occ_last_error(void);
+
+/* OCC_VERSION of the built library. */
+int occ_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OCC_H_ */

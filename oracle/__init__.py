@@ -28,7 +28,8 @@ closed forms, invariants, brute force on tiny inputs, finite differences, and
 the values printed in Table 4 (``tests/golden/``).  No function is unpinned.
 """
 
-from .loss import LossParams, token_logprob, token_terms, decoupled_loss, FLAG_IN_BAND, \
+from .loss import LossParams, token_logprob, token_terms, decoupled_loss, softmax_grad_rows, \
+    FLAG_IN_BAND, \
     FLAG_CLIPPED, FLAG_ACTIVE, FLAG_VALID  # noqa: F401
 from .ewma import EwmaState, ewma_coefficients, ewma_update, ewma_closed_form, \
     beta_for_window, center_of_mass  # noqa: F401

@@ -1,0 +1,58 @@
+// Status strings, per-thread error messages and device queries of the occ C ABI.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include "occ_internal.h"
+
+namespace occ {
+
+static thread_local char g_msg[512] = "";
+
+occ_status fail(occ_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+void clear_error() { g_msg[0] = '\0'; }
+
+occ_status check_launch(const char* what) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(OCC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+  return OCC_OK;
+}
+
+int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  if (dev >= 0 && dev < 64 && cached[dev]) return cached[dev];
+  int n = 1;
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  if (dev >= 0 && dev < 64) cached[dev] = n;
+  return n;
+}
+
+}  // namespace occ
+
+extern "C" {
+
+const char* occ_status_string(occ_status s) {
+  switch (s) {
+    case OCC_OK: return "ok";
+    case OCC_ERR_INVALID_ARG: return "invalid argument";
+    case OCC_ERR_UNSUPPORTED: return "unsupported dtype or size";
+    case OCC_ERR_MISALIGNED: return "misaligned pointer";
+    case OCC_ERR_CUDA: return "CUDA error";
+    case OCC_ERR_WORKSPACE: return "workspace missing or too small";
+  }
+  return "unknown status";
+}
+
+const char* occ_last_error(void) { return occ::g_msg; }
+
+int occ_version(void) { return OCC_VERSION; }
+
+}  // extern "C"

@@ -1,0 +1,237 @@
+// Device building blocks shared by the occ kernels (sm_103a).
+//
+// The row statistic every kernel needs is the log-partition function
+// lse = log sum_v exp(z_v) of a logits row (Eq. 1 ratios are quotients of
+// softmax probabilities).  Each thread keeps an online pair (c, s) in base-2
+// scaled units: s = sum 2^(z_v * L - c) with L = float(log2 e).  The reference
+// exponent c only moves when a new value exceeds it by more than kRescale
+// (lazy rescaling), so the inner loop is one FFMA, one MUFU.EX2 and one FADD
+// per element.  Partials are merged with one accurate exp2f per thread and a
+// compensated (two-float) tree sum, and the row epilogue runs in float64.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "occ.h"
+#include "occ_internal.h"
+
+namespace occ {
+
+constexpr float kLog2e = 1.4426950408889634f;  // float(log2 e)
+constexpr float kRescale = 64.f;               // lazy-rescale margin (base-2 exponent units)
+
+// ---------------------------------------------------------------- PTX helpers
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Streaming 16-byte load: bypass L1, 256-byte L2 prefetch granularity.
+__device__ __forceinline__ uint4 ld_stream_v4(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+// Streaming (evict-first) 16-byte store.
+__device__ __forceinline__ void st_stream_v4(void* p, uint4 v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+
+// Round-to-nearest-even float -> bf16 scalar store to global memory.
+__device__ __forceinline__ void st_bf16(void* p, float x) {
+  unsigned short h;
+  asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(x));
+  asm volatile("st.global.u16 [%0], %1;" ::"l"(p), "h"(h) : "memory");
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Scalar element access for the two input types.
+template <typename T>
+struct Elem;
+template <>
+struct Elem<float> {
+  static constexpr int kVec = 4;  // elements per 16-byte vector
+  __device__ __forceinline__ static float load(const float* p) { return *(const volatile float*)p; }
+  __device__ __forceinline__ static void put(float* p, float x) { *p = x; }
+  __device__ __forceinline__ static void unpack(const uint4& r, float (&x)[4]) {
+    x[0] = __uint_as_float(r.x);
+    x[1] = __uint_as_float(r.y);
+    x[2] = __uint_as_float(r.z);
+    x[3] = __uint_as_float(r.w);
+  }
+};
+struct bf16_t {
+  uint16_t bits;
+};
+template <>
+struct Elem<bf16_t> {
+  static constexpr int kVec = 8;
+  __device__ __forceinline__ static float load(const bf16_t* p) {
+    unsigned short b;
+    asm volatile("ld.global.u16 %0, [%1];" : "=h"(b) : "l"(p));
+    return __uint_as_float(((uint32_t)b) << 16);
+  }
+  // Stores a value that is exactly representable in bf16 (its top 16 bits).
+  __device__ __forceinline__ static void put(bf16_t* p, float x) {
+    p->bits = (uint16_t)(__float_as_uint(x) >> 16);
+  }
+  __device__ __forceinline__ static void unpack(const uint4& r, float (&x)[8]) {
+    x[0] = bf16_lo(r.x); x[1] = bf16_hi(r.x);
+    x[2] = bf16_lo(r.y); x[3] = bf16_hi(r.y);
+    x[4] = bf16_lo(r.z); x[5] = bf16_hi(r.z);
+    x[6] = bf16_lo(r.w); x[7] = bf16_hi(r.w);
+  }
+};
+
+// ------------------------------------------------------- online log-sum-exp
+
+struct LseAcc {
+  float c;  // reference exponent, base-2 scaled units (-inf: nothing finite seen)
+  float s;  // sum of 2^(z L - c)
+};
+
+__device__ __forceinline__ void acc_init(LseAcc& a) {
+  a.c = -INFINITY;
+  a.s = 0.f;
+}
+
+template <int N>
+__device__ __forceinline__ void acc_add(LseAcc& a, const float (&x)[N]) {
+  float m = x[0];
+#pragma unroll
+  for (int j = 1; j < N; ++j) m = fmaxf(m, x[j]);
+  const float ms = m * kLog2e;
+  if (ms > a.c + kRescale) {  // also taken by the first finite vector (c = -inf)
+    a.s *= exp2f(a.c - ms);
+    a.c = ms;
+  }
+  if (a.c != -INFINITY) {
+    float t = 0.f;
+#pragma unroll
+    for (int j = 0; j < N; ++j) t += ex2_approx(fmaf(x[j], kLog2e, -a.c));
+    a.s += t;
+  }
+}
+
+// ------------------------------------------------------------ reductions
+
+// Two-float compensated addition (Knuth TwoSum on the high parts).
+__device__ __forceinline__ float2 pair_add(float2 a, float2 b) {
+  const float s = a.x + b.x;
+  const float bp = s - a.x;
+  const float e = (a.x - (s - bp)) + (b.x - bp);
+  return make_float2(s, e + (a.y + b.y));
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float2 warp_pair_sum(float2 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    float2 w;
+    w.x = __shfl_xor_sync(0xffffffffu, v.x, o);
+    w.y = __shfl_xor_sync(0xffffffffu, v.y, o);
+    v = pair_add(v, w);
+  }
+  return v;
+}
+
+// Shared scratch for block reductions (one slot per warp).
+struct RedScratch {
+  float m[32];
+  float2 s[32];
+  float bc;
+};
+
+// Merges the per-thread (c, s) of a block.  Result (C, S) is valid in thread 0:
+// sum over the block of 2^(z L - C) = S.x + S.y.  Deterministic order.
+template <int NT>
+__device__ __forceinline__ void block_lse(const LseAcc& a, RedScratch& r, float& C, float2& S) {
+  constexpr int NW = NT / 32;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  float m = warp_max(a.c);
+  if (lane == 0) r.m[wid] = m;
+  __syncthreads();
+  if (wid == 0) {
+    float v = lane < NW ? r.m[lane] : -INFINITY;
+    v = warp_max(v);
+    if (lane == 0) r.bc = v;
+  }
+  __syncthreads();
+  const float Cb = r.bc;
+  float2 v = make_float2((a.c == -INFINITY) ? 0.f : a.s * exp2f(a.c - Cb), 0.f);
+  v = warp_pair_sum(v);
+  if (lane == 0) r.s[wid] = v;
+  __syncthreads();
+  if (wid == 0) {
+    float2 w = lane < NW ? r.s[lane] : make_float2(0.f, 0.f);
+    w = warp_pair_sum(w);
+    if (lane == 0) S = w;
+  }
+  C = Cb;
+}
+
+// Row epilogue in float64: lse from the merged (C, S).  The terms were
+// 2^(z L - C) with L = float(log2 e); dividing the base-2 result by that same
+// L keeps the error at float(log2 e)'s relative error times the row entropy.
+__device__ __forceinline__ double lse_from(float C, float2 S) {
+  if (!(S.x > 0.f)) return (S.x == 0.f) ? -INFINITY : (double)NAN;
+  int e;
+  const float f = frexpf(S.x, &e);  // S.x = f 2^e, f in [0.5, 1)
+  const double l2 = (double)C + (double)e + (double)log2f(f) +
+                    (double)(S.y / S.x) * 1.4426950408889634;
+  return l2 / (double)kLog2e;
+}
+
+// ------------------------------------------------------------- cluster PTX
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Reads a float4 from the shared memory of CTA `rank` of this cluster.
+__device__ __forceinline__ float4 ld_dsmem_f4(const void* local_smem_ptr, uint32_t rank) {
+  uint32_t local = (uint32_t)__cvta_generic_to_shared(local_smem_ptr);
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(rank));
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(remote)
+               : "memory");
+  return v;
+}
+
+}  // namespace occ

@@ -1,0 +1,31 @@
+// Host-side helpers shared by the occ translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "occ.h"
+
+namespace occ {
+
+// Records a printf-style message for occ_last_error() and returns `s`.
+occ_status fail(occ_status s, const char* fmt, ...);
+// Clears the message of the calling thread.
+void clear_error();
+// Maps a CUDA error (after a launch) to OCC_ERR_CUDA with a message.
+occ_status check_launch(const char* what);
+
+inline bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Byte ranges [a, a+na) and [b, b+nb) intersect.
+inline bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+  return na && nb && x < y + nb && y < x + na;
+}
+
+inline size_t dtype_size(occ_dtype dt) { return dt == OCC_BF16 ? 2 : 4; }
+
+// Multiprocessor count of the current device (cached per device).
+int sm_count();
+
+}  // namespace occ

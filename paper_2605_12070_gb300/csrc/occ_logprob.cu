@@ -1,0 +1,144 @@
+// K1: vocabulary-streaming log-sum-exp and sampled-token log-probability.
+//
+// log pi(y_t) = z[t, y_t] - log sum_v exp(z[t, v]) for each row t: the per-token
+// factors of the ratios in Eq. 1 (used for pi_old, pi_prox of Eq. 5 or
+// pi_async of Table 1).  One CTA streams one row with 16-byte coalesced loads,
+// U vectors in flight per thread, and keeps an online (c, s) pair per thread;
+// nothing is staged in shared memory because each element is used once.
+// HBM traffic is the logits row once: V * sizeof(T) bytes per token.
+#include "occ_common.cuh"
+
+namespace occ {
+
+constexpr int kK1Threads = 512;
+constexpr int kK1Unroll = 8;
+
+template <typename Tin, int NT, int U>
+__global__ void __launch_bounds__(NT, 2)
+    k1_logprob_vec(const Tin* __restrict__ logits, int64_t T, int64_t V, int64_t ld,
+                   const int32_t* __restrict__ ids, float* __restrict__ logp,
+                   float* __restrict__ lse_out) {
+  constexpr int VEC = Elem<Tin>::kVec;
+  __shared__ RedScratch red;
+  const int64_t nvec = V / VEC;
+  const int64_t tail0 = nvec * VEC;
+  for (int64_t row = blockIdx.x; row < T; row += gridDim.x) {
+    const Tin* z = logits + row * ld;
+    int id = 0;
+    float zy = 0.f;
+    if (threadIdx.x == 0) {
+      id = ids[row];
+      if (id >= 0 && id < V) zy = Elem<Tin>::load(z + id);
+    }
+    LseAcc acc;
+    acc_init(acc);
+    const uint4* zv = reinterpret_cast<const uint4*>(z);
+    int64_t i = threadIdx.x;
+    for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
+      uint4 r[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) r[u] = ld_stream_v4(zv + i + u * NT);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        float x[VEC];
+        Elem<Tin>::unpack(r[u], x);
+        acc_add(acc, x);
+      }
+    }
+    for (; i < nvec; i += NT) {
+      float x[VEC];
+      Elem<Tin>::unpack(ld_stream_v4(zv + i), x);
+      acc_add(acc, x);
+    }
+    if ((int64_t)threadIdx.x < V - tail0) {
+      float x[1] = {Elem<Tin>::load(z + tail0 + threadIdx.x)};
+      acc_add(acc, x);
+    }
+    float C;
+    float2 S;
+    block_lse<NT>(acc, red, C, S);
+    if (threadIdx.x == 0) {
+      const double l = lse_from(C, S);
+      logp[row] = (id >= 0 && id < V) ? (float)((double)zy - l) : __int_as_float(0x7fc00000);
+      if (lse_out) lse_out[row] = (float)l;
+    }
+    __syncthreads();
+  }
+}
+
+// Any alignment: element loads, consecutive threads on consecutive columns.
+template <typename Tin, int NT>
+__global__ void __launch_bounds__(NT)
+    k1_logprob_scalar(const Tin* __restrict__ logits, int64_t T, int64_t V, int64_t ld,
+                      const int32_t* __restrict__ ids, float* __restrict__ logp,
+                      float* __restrict__ lse_out) {
+  __shared__ RedScratch red;
+  for (int64_t row = blockIdx.x; row < T; row += gridDim.x) {
+    const Tin* z = logits + row * ld;
+    int id = 0;
+    float zy = 0.f;
+    if (threadIdx.x == 0) {
+      id = ids[row];
+      if (id >= 0 && id < V) zy = Elem<Tin>::load(z + id);
+    }
+    LseAcc acc;
+    acc_init(acc);
+    for (int64_t v0 = threadIdx.x; v0 < V; v0 += 8 * (int64_t)NT) {
+      float x[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int64_t v = v0 + (int64_t)j * NT;
+        x[j] = v < V ? Elem<Tin>::load(z + v) : -INFINITY;
+      }
+      acc_add(acc, x);
+    }
+    float C;
+    float2 S;
+    block_lse<NT>(acc, red, C, S);
+    if (threadIdx.x == 0) {
+      const double l = lse_from(C, S);
+      logp[row] = (id >= 0 && id < V) ? (float)((double)zy - l) : __int_as_float(0x7fc00000);
+      if (lse_out) lse_out[row] = (float)l;
+    }
+    __syncthreads();
+  }
+}
+
+template <typename Tin>
+static void launch_k1(const void* logits, int64_t T, int64_t V, int64_t ld, const int32_t* ids,
+                      float* logp, float* lse, bool vec, cudaStream_t s) {
+  const unsigned grid = (unsigned)(T < 0x7fffffffLL ? T : 0x7fffffffLL);
+  if (vec)
+    k1_logprob_vec<Tin, kK1Threads, kK1Unroll><<<grid, kK1Threads, 0, s>>>(
+        (const Tin*)logits, T, V, ld, ids, logp, lse);
+  else
+    k1_logprob_scalar<Tin, kK1Threads><<<grid, kK1Threads, 0, s>>>((const Tin*)logits, T, V, ld,
+                                                                    ids, logp, lse);
+}
+
+}  // namespace occ
+
+using namespace occ;
+
+extern "C" occ_status occ_token_logprob(const void* logits, occ_dtype dt, int64_t T, int64_t V,
+                                        int64_t ld, const int32_t* ids, float* logp_out,
+                                        float* lse_out, void* stream) {
+  clear_error();
+  if (dt != OCC_F32 && dt != OCC_BF16) return fail(OCC_ERR_UNSUPPORTED, "dtype %d", (int)dt);
+  if (T < 0 || V < 1 || ld < V)
+    return fail(OCC_ERR_INVALID_ARG, "need T >= 0, V >= 1, ld >= V (T=%lld V=%lld ld=%lld)",
+                (long long)T, (long long)V, (long long)ld);
+  if (T == 0) return OCC_OK;
+  if (!logits || !ids || !logp_out) return fail(OCC_ERR_INVALID_ARG, "null logits/ids/logp_out");
+  const size_t es = dtype_size(dt);
+  if (!aligned(logits, es) || !aligned(ids, 4) || !aligned(logp_out, 4) ||
+      (lse_out && !aligned(lse_out, 4)))
+    return fail(OCC_ERR_MISALIGNED, "arrays must be aligned to their element size");
+  const bool vec = aligned(logits, 16) && ((ld * (int64_t)es) % 16 == 0);
+  cudaStream_t s = (cudaStream_t)stream;
+  if (dt == OCC_BF16)
+    launch_k1<bf16_t>(logits, T, V, ld, ids, logp_out, lse_out, vec, s);
+  else
+    launch_k1<float>(logits, T, V, ld, ids, logp_out, lse_out, vec, s);
+  return check_launch("occ_token_logprob");
+}

@@ -1,0 +1,258 @@
+"""Thin ctypes binding of the occ C ABI (include/occ.h) for torch tensors.
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels of ``libocc.so``.  The functions carry the C names.  Tensors must be
+CUDA tensors; outputs not supplied by the caller are allocated with
+``torch.empty`` on the input's device.  Calls are asynchronous on the current
+torch stream unless ``stream`` (a ``torch.cuda.Stream``) is given.
+
+There is no CPU fallback: if the library is missing or a tensor is not on a
+CUDA device, the call raises.
+"""
+
+import ctypes
+import os
+import struct
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libocc.so")
+
+OCC_OK = 0
+OCC_F32, OCC_BF16 = 0, 1
+FLAG_IN_BAND, FLAG_CLIPPED, FLAG_ACTIVE, FLAG_VALID = 1, 2, 4, 8
+DATA_ERR_BAD_ID = 1
+
+LOSS_STATS_BYTES = 64     # sizeof(occ_loss_stats)
+EWMA_STATE_BYTES = 40     # sizeof(occ_ewma_state)
+_STATS_FMT = "<2d5q2i"
+_STATE_FMT = "<3d4i"
+
+# Every symbol declared in include/occ.h.
+EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_fwd_bwd",
+           "occ_ewma_update", "occ_ewma_state_init", "occ_status_string", "occ_last_error",
+           "occ_version")
+
+
+class OccError(RuntimeError):
+    pass
+
+
+class LossParams(ctypes.Structure):
+    """Mirror of occ_loss_params (host struct)."""
+    _fields_ = [("rd_lo", ctypes.c_double), ("rd_hi", ctypes.c_double),
+                ("eps_low", ctypes.c_double), ("eps_high", ctypes.c_double),
+                ("grad_scale", ctypes.c_double), ("denom", ctypes.c_int64),
+                ("rd_weight", ctypes.c_int32), ("dlogits_f32", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def lib():
+    """Loads libocc.so once; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise OccError(f"{LIB_PATH} is not built; run `python -m paper_2605_12070_gb300.build` "
+                       "or __graft_entry__.build()")
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i64, i32, dbl = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_double
+    L.occ_token_logprob.argtypes = [vp, i32, i64, i64, i64, vp, vp, vp, vp]
+    L.occ_token_logprob.restype = i32
+    L.occ_loss_workspace_bytes.argtypes = [i64, i64]
+    L.occ_loss_workspace_bytes.restype = ctypes.c_size_t
+    L.occ_decoupled_loss_fwd_bwd.argtypes = [vp, i32, i64, i64, i64, vp, vp, vp, vp, vp,
+                                             ctypes.POINTER(LossParams), vp, vp, vp, i64, vp, vp,
+                                             ctypes.c_size_t, vp]
+    L.occ_decoupled_loss_fwd_bwd.restype = i32
+    L.occ_ewma_update.argtypes = [vp, vp, i64, dbl, vp, vp, dbl, i32, i32, vp]
+    L.occ_ewma_update.restype = i32
+    L.occ_ewma_state_init.argtypes = [vp, dbl, vp]
+    L.occ_ewma_state_init.restype = i32
+    L.occ_status_string.argtypes = [i32]
+    L.occ_status_string.restype = ctypes.c_char_p
+    L.occ_last_error.argtypes = []
+    L.occ_last_error.restype = ctypes.c_char_p
+    L.occ_version.argtypes = []
+    L.occ_version.restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def _check(rc, what):
+    if rc != OCC_OK:
+        L = lib()
+        raise OccError(f"{what}: {L.occ_status_string(rc).decode()} "
+                       f"({L.occ_last_error().decode()})")
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream, device):
+    s = stream if stream is not None else torch.cuda.current_stream(device)
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _cuda(*ts):
+    for t in ts:
+        if t is not None and not t.is_cuda:
+            raise OccError("occ kernels need CUDA tensors (no CPU fallback)")
+
+
+def _dtype_code(t):
+    if t.dtype == torch.bfloat16:
+        return OCC_BF16
+    if t.dtype == torch.float32:
+        return OCC_F32
+    raise OccError(f"unsupported logits dtype {t.dtype}")
+
+
+def _rows(logits):
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise OccError("logits must be a 2-D tensor with unit column stride")
+    return logits.shape[0], logits.shape[1], logits.stride(0)
+
+
+def occ_token_logprob(logits, ids, logp_out=None, lse_out=None, want_lse=False, stream=None):
+    """log pi(y_t) (and optionally lse) for each row of ``logits`` [T, V]."""
+    _cuda(logits, ids, logp_out, lse_out)
+    T, V, ld = _rows(logits)
+    if logp_out is None:
+        logp_out = torch.empty(T, dtype=torch.float32, device=logits.device)
+    if lse_out is None and want_lse:
+        lse_out = torch.empty(T, dtype=torch.float32, device=logits.device)
+    rc = lib().occ_token_logprob(_ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids),
+                                 _ptr(logp_out), _ptr(lse_out), _stream(stream, logits.device))
+    _check(rc, "occ_token_logprob")
+    return logp_out, lse_out
+
+
+def occ_loss_workspace_bytes(T, V):
+    return int(lib().occ_loss_workspace_bytes(int(T), int(V)))
+
+
+def new_loss_stats(device):
+    return torch.zeros(LOSS_STATS_BYTES, dtype=torch.uint8, device=device)
+
+
+def new_workspace(T, V, device):
+    return torch.empty(occ_loss_workspace_bytes(T, V), dtype=torch.uint8, device=device)
+
+
+@dataclass
+class LossStats:
+    loss_sum: float
+    loss: float
+    n_valid: int
+    n_rd_out: int
+    n_clipped: int
+    n_active: int
+    denom: int
+    err: int
+
+    @property
+    def rho(self):
+        """Train-Infer Mask value of Sec. 5.2: fraction of valid tokens kept active."""
+        return self.n_active / self.n_valid if self.n_valid else float("nan")
+
+
+def decode_loss_stats(t):
+    v = struct.unpack(_STATS_FMT, bytes(t.detach().to("cpu").numpy().tobytes()))
+    return LossStats(*v[:8])
+
+
+def occ_decoupled_loss_fwd_bwd(logits, ids, logp_old, logp_mu, adv, loss_mask=None, *,
+                               rd_lo, rd_hi, eps_low, eps_high, rd_weight=1, grad_scale=1.0,
+                               denom=0, dlogits_f32=False, dlogits="new", logp_out=None,
+                               flags_out=None, want_logp=True, want_flags=True, stats=None,
+                               workspace=None, stream=None):
+    """The decoupled PPO loss over ``logits`` [T, V] and its gradient.
+
+    ``dlogits``: "new" (allocate), None (forward only), "inplace" (overwrite
+    ``logits``), or a tensor [T, >=V].  Returns a dict with 'stats' (raw
+    device bytes), 'dlogits', 'logp', 'flags'.
+    """
+    _cuda(logits, ids, logp_old, logp_mu, adv, loss_mask)
+    T, V, ld = _rows(logits)
+    dev = logits.device
+    out_dtype = torch.float32 if (dlogits_f32 or logits.dtype == torch.float32) else logits.dtype
+    if isinstance(dlogits, str):
+        if dlogits == "new":
+            dlogits = torch.empty((T, V), dtype=out_dtype, device=dev)
+        elif dlogits == "inplace":
+            dlogits = logits
+        else:
+            raise OccError(f"dlogits={dlogits!r}")
+    if dlogits is not None:
+        _cuda(dlogits)
+        if dlogits.dim() != 2 or dlogits.stride(1) != 1 or dlogits.dtype != out_dtype:
+            raise OccError("dlogits must be 2-D, unit column stride, dtype " + str(out_dtype))
+    ld_grad = dlogits.stride(0) if dlogits is not None else 0
+    if logp_out is None and want_logp:
+        logp_out = torch.empty(T, dtype=torch.float32, device=dev)
+    if flags_out is None and want_flags:
+        flags_out = torch.empty(T, dtype=torch.uint8, device=dev)
+    if stats is None:
+        stats = new_loss_stats(dev)
+    if workspace is None:
+        workspace = new_workspace(T, V, dev)
+    p = LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
+                   float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)))
+    rc = lib().occ_decoupled_loss_fwd_bwd(
+        _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
+        _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
+        _ptr(dlogits), ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(),
+        _stream(stream, dev))
+    _check(rc, "occ_decoupled_loss_fwd_bwd")
+    return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "flags": flags_out}
+
+
+def new_ewma_state(device, w0=0.0, stream=None):
+    st = torch.zeros(EWMA_STATE_BYTES, dtype=torch.uint8, device=device)
+    occ_ewma_state_init(st, w0, stream)
+    return st
+
+
+def occ_ewma_state_init(state, w0, stream=None):
+    _cuda(state)
+    _check(lib().occ_ewma_state_init(_ptr(state), float(w0), _stream(stream, state.device)),
+           "occ_ewma_state_init")
+
+
+@dataclass
+class EwmaState:
+    w: float
+    coef_a: float
+    coef_b: float
+    streak: int
+    n_resets: int
+    last_reset: int
+
+
+def decode_ewma_state(t):
+    v = struct.unpack(_STATE_FMT, bytes(t.detach().to("cpu").numpy().tobytes()))
+    return EwmaState(*v[:6])
+
+
+def occ_ewma_update(theta_prox, theta, beta, state, stats=None, tau=0.9, min_streak=1,
+                    force_reset=False, stream=None):
+    """theta_prox <- revised PPO-EWMA step toward theta (in place)."""
+    _cuda(theta_prox, theta, state, stats)
+    if theta_prox.dtype != torch.float32 or theta.dtype != torch.float32:
+        raise OccError("EWMA buffers must be float32")
+    if not (theta_prox.is_contiguous() and theta.is_contiguous()):
+        raise OccError("EWMA buffers must be contiguous")
+    n = theta_prox.numel()
+    if theta.numel() != n:
+        raise OccError("theta_prox and theta differ in size")
+    rc = lib().occ_ewma_update(_ptr(theta_prox), _ptr(theta), n, float(beta), _ptr(state),
+                               _ptr(stats), float(tau), int(min_streak), int(bool(force_reset)),
+                               _stream(stream, theta_prox.device))
+    _check(rc, "occ_ewma_update")
+    return theta_prox

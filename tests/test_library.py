@@ -1,0 +1,85 @@
+"""Host-side checks of the C-ABI library that need no GPU.
+
+The library must load, export every entry point include/occ.h declares, and
+reject invalid calls on the host before touching the device.
+"""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2605_12070_gb300 import build, occ
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return occ.lib()
+
+
+def _declared_symbols():
+    names = set()
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", f)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(occ_[a-z0-9_]+)\s*\(", src))
+    return names
+
+
+def test_every_declared_symbol_is_exported(L):
+    declared = _declared_symbols()
+    assert {"occ_token_logprob", "occ_decoupled_loss_fwd_bwd", "occ_ewma_update"} <= declared
+    for name in declared:
+        assert hasattr(L, name), name
+    assert declared <= set(occ.EXPORTS)
+
+
+def test_version_and_status_strings(L):
+    assert L.occ_version() == 1
+    assert L.occ_status_string(0) == b"ok"
+    assert L.occ_status_string(5).startswith(b"workspace")
+
+
+def test_host_validation_without_gpu(L):
+    null = ctypes.c_void_p(0)
+    # V = 0 is rejected before any CUDA call
+    rc = L.occ_token_logprob(null, 0, 4, 0, 0, null, null, null, null)
+    assert rc == 1 and b"V >= 1" in L.occ_last_error()
+    # T = 0 is a no-op
+    assert L.occ_token_logprob(null, 1, 0, 10, 10, null, null, null, null) == 0
+    # bad dtype
+    assert L.occ_token_logprob(null, 7, 1, 10, 10, null, null, null, null) == 2
+    # inverted band
+    p = occ.LossParams(2.0, 1.0, 0.2, 0.28, 1.0, 0, 1, 0)
+    rc = L.occ_decoupled_loss_fwd_bwd(null, 1, 1, 8, 8, null, null, null, null, null,
+                                      ctypes.byref(p), null, null, null, 0, null, null, 0, null)
+    assert rc == 1
+    # missing workspace
+    p = occ.LossParams(0.5, 2.0, 0.2, 0.28, 1.0, 0, 1, 0)
+    stats = ctypes.create_string_buffer(64)
+    rc = L.occ_decoupled_loss_fwd_bwd(null, 1, 1, 8, 8, null, null, null, null, null,
+                                      ctypes.byref(p), null, null, null, 0,
+                                      ctypes.cast(stats, ctypes.c_void_p), null, 0, null)
+    assert rc == 5
+    # EWMA: beta out of range, min_streak < 1
+    st = ctypes.create_string_buffer(48)
+    stp = ctypes.cast(st, ctypes.c_void_p)
+    assert L.occ_ewma_update(null, null, 0, 1.5, stp, null, 0.9, 1, 0, null) == 1
+    assert L.occ_ewma_update(null, null, 0, 0.5, stp, null, 0.9, 0, 0, null) == 1
+
+
+def test_workspace_size_grows_with_tokens(L):
+    a = occ.occ_loss_workspace_bytes(0, 151936)
+    b = occ.occ_loss_workspace_bytes(65536, 151936)
+    assert 0 < a < b and b >= 65536 * 5 and b % 256 == 0
+
+
+def test_no_cpu_fallback():
+    import torch
+    with pytest.raises(occ.OccError, match="CUDA"):
+        occ.occ_token_logprob(torch.zeros(2, 4), torch.zeros(2, dtype=torch.int32))
