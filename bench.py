@@ -43,8 +43,9 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-rows", type=int, default=96)
-    ap.add_argument("--cpu-params", type=int, default=1 << 25)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--tau", type=float, default=0.5)
+    ap.add_argument("--tokens", type=int, default=None, help="resize T (profiling runs only)")
     return ap.parse_args()
 
 
@@ -192,21 +193,35 @@ def oracle_sample_times(batch, rows, n_params, threads):
     return t_rows, t_par
 
 
-def cpu_baseline(batch, n_params_full, rows_n, params_n):
+def cpu_baseline(batch, n_params_full, seconds):
+    """Times the oracle, as it stands, on growing row chunks of the batch and an
+    EWMA sample until about `seconds` of CPU work, then scales to one step."""
     import numpy as np
 
     from oracle.rows import host_cores
     threads = host_cores()
     rng = np.random.default_rng(0)
     valid = np.nonzero(batch.mask.cpu().numpy())[0] if batch.mask is not None else np.arange(batch.T)
-    rows = np.sort(rng.choice(valid, size=min(rows_n, valid.size), replace=False))
-    t_rows, t_par = oracle_sample_times(batch, rows, params_n, threads)
-    step_s = batch.T * t_rows / rows.size + n_params_full * t_par / params_n
+    order = rng.permutation(valid)
+    t_rows = t_par = 0.0
+    n_rows = n_par = 0
+    chunk = 4 * threads
+    while t_rows < 0.7 * seconds and n_rows < order.size:
+        rows = np.sort(order[n_rows:n_rows + chunk])
+        tr, _ = oracle_sample_times(batch, rows, 0, threads)
+        t_rows += tr
+        n_rows += rows.size
+    par_chunk = 1 << 24
+    while t_par < 0.3 * seconds and n_par < (1 << 30):
+        _, tp = oracle_sample_times(batch, np.zeros(0, dtype=np.int64), par_chunk, threads)
+        t_par += tp
+        n_par += par_chunk
+    step_s = batch.T * t_rows / n_rows + n_params_full * t_par / n_par
     return {
-        "value": batch.T / step_s, "unit": "tokens/s", "cores": threads, "kind": "oracle",
-        "sample": (f"float64 numpy oracle on {rows.size} valid tokens of the T={batch.T}, "
-                   f"V={batch.V} batch ({t_rows:.2f} s) and {params_n} EWMA elements "
-                   f"({t_par:.2f} s), scaled to T tokens + {n_params_full} parameters per step"),
+        "value": round(batch.T / step_s, 3), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+        "sample": (f"float64 numpy oracle on {n_rows} valid tokens of the T={batch.T}, "
+                   f"V={batch.V} batch ({t_rows:.1f} s) and {n_par} EWMA elements "
+                   f"({t_par:.1f} s), scaled to T tokens + {n_params_full} parameters per step"),
         "seconds": round(t_rows + t_par, 2),
     }
 
@@ -234,7 +249,7 @@ def main():
     from paper_2605_12070_gb300 import dp, occ
     from paper_2605_12070_gb300.workloads import make_ewma_buffers, make_loss_batch
 
-    batch = make_loss_batch(WORKLOAD, seed=rank, device=dev)
+    batch = make_loss_batch(WORKLOAD, T=args.tokens, seed=rank, device=dev)
     T, V = batch.T, batch.V
     n_valid = int(batch.mask.sum().item())
 
@@ -267,7 +282,7 @@ def main():
             dp.allreduce_loss_stats(stats)
         if ev is not None:
             ev[2].record(stream)
-        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=0.9)
+        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=args.tau)
         if ev is not None:
             ev[3].record(stream)
 
@@ -283,6 +298,7 @@ def main():
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid).replace("GPU-", "")
     except Exception:
         gpu_id = local
+    resets_before = occ.decode_ewma_state(state).n_resets
     clocks = ClockSampler(gpu_id)
     clocks.start()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
@@ -311,7 +327,10 @@ def main():
     traffic = ncu_traffic()
     bytes_k1 = T * V * 2 + T * 8
     bytes_k2 = n_valid * V * 2 + T * V * 2 + T * 37
-    bytes_k3 = args.ewma_n * 12
+    resets = occ.decode_ewma_state(state).n_resets - resets_before
+    # a regular update reads theta_prox and theta and writes theta_prox; a reset copies theta
+    bytes_k3 = args.ewma_n * (12 * (args.steps - resets) + 8 * resets) // args.steps
+    st_last = occ.decode_loss_stats(stats)
     kern = {
         "k1_token_logprob": (k1, bytes_k1, T),
         "k2_decoupled_loss_fwd_bwd": (k2, bytes_k2, T),
@@ -350,6 +369,8 @@ def main():
             "T": T, "V": V, "ewma_params": args.ewma_n, "logits_dtype": "bf16",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": "inputs larger than L2 (40 GB logits, 61 GB EWMA buffers): no flush",
+            "rd_band": [batch.rd_lo, batch.rd_hi], "eps": [batch.eps_low, batch.eps_high],
+            "tau": args.tau, "rho": round(st_last.rho, 5), "ewma_resets_timed": resets,
         },
         "roofline": dict(roof[dominant], kernel=dominant),
         "kernels": roof,
@@ -359,7 +380,7 @@ def main():
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(batch, args.ewma_n, args.cpu_rows, args.cpu_params)
+        line["cpu_baseline"] = cpu_baseline(batch, args.ewma_n, args.cpu_seconds)
     if not args.no_e2e:
         line["e2e"] = run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits,
                               logp, flags, denom, world, dev)
@@ -411,7 +432,7 @@ def run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits, l
                                        stats=stats, workspace=ws)
         if world > 1:
             dp.allreduce_loss_stats(stats)
-        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=0.9)
+        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=args.tau)
         stats_h.copy_(stats, non_blocking=True)
 
     e2e_step()

@@ -32,8 +32,8 @@ _STATE_FMT = "<3d4i"
 
 # Every symbol declared in include/occ.h.
 EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_fwd_bwd",
-           "occ_ewma_update", "occ_ewma_state_init", "occ_status_string", "occ_last_error",
-           "occ_version")
+           "occ_ewma_update", "occ_ewma_state_init",
+           "occ_status_string", "occ_last_error", "occ_version")
 
 
 class OccError(RuntimeError):
