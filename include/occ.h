@@ -160,6 +160,37 @@ occ_status occ_decoupled_loss_fwd_bwd(const void* logits, occ_dtype dt, int64_t 
                                       size_t ws_bytes, void* stream);
 
 /*
+ * occ_decoupled_loss_fwd_bwd_noalloc -- occ_decoupled_loss_fwd_bwd without a
+ * caller-supplied workspace.  (The paper has no counterpart: this is an
+ * interface convenience.)
+ *
+ * For callers that cannot allocate device memory themselves -- for instance a
+ * plain C plugin running inside a framework whose caching allocator owns all
+ * of the GPU's memory, or a loop that must not call cudaMalloc/cudaFree
+ * because those can synchronize the device.  Arguments, results and
+ * validation are those of occ_decoupled_loss_fwd_bwd minus (workspace,
+ * ws_bytes).  Neither the caller nor the library allocates anything: the
+ * scratch is a fixed 4 MiB array in the library's device globals, which
+ * every GPU that loads the library holds until the process exits.
+ *   - T may be at most OCC_NOALLOC_MAX_TOKENS; larger batches are rejected
+ *     with OCC_ERR_UNSUPPORTED before anything is launched.
+ *   - The first call on a device (with that device current) looks up the
+ *     array's device address; make that first call before any stream capture.
+ *   - All calls share the one array: calls that may overlap on the GPU (other
+ *     streams, other host threads) race with each other.  Serialise them.
+ *     Every call writes all the scratch it later reads, so nothing left over
+ *     from an earlier call affects the result.
+ */
+#define OCC_NOALLOC_MAX_TOKENS 786432
+occ_status occ_decoupled_loss_fwd_bwd_noalloc(const void* logits, occ_dtype dt, int64_t T,
+                                              int64_t V, int64_t ld, const int32_t* ids,
+                                              const float* logp_old, const float* logp_mu,
+                                              const float* adv, const uint8_t* loss_mask,
+                                              const occ_loss_params* p, float* logp_out,
+                                              uint8_t* flags_out, void* dlogits, int64_t ld_grad,
+                                              occ_loss_stats* stats, void* stream);
+
+/*
  * occ_ewma_update -- revised PPO-EWMA step on flat float32 parameters.
  *
  * App. B recursion: w <- 1 + beta w, theta_prox <- a theta_prox + b theta with

@@ -32,7 +32,7 @@ _STATE_FMT = "<3d4i"
 
 # Every symbol declared in include/occ.h.
 EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_fwd_bwd",
-           "occ_ewma_update", "occ_ewma_state_init",
+           "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update", "occ_ewma_state_init",
            "occ_status_string", "occ_last_error", "occ_version")
 
 
@@ -69,6 +69,10 @@ def lib():
                                              ctypes.POINTER(LossParams), vp, vp, vp, i64, vp, vp,
                                              ctypes.c_size_t, vp]
     L.occ_decoupled_loss_fwd_bwd.restype = i32
+    L.occ_decoupled_loss_fwd_bwd_noalloc.argtypes = [vp, i32, i64, i64, i64, vp, vp, vp, vp, vp,
+                                                     ctypes.POINTER(LossParams), vp, vp, vp, i64,
+                                                     vp, vp]
+    L.occ_decoupled_loss_fwd_bwd_noalloc.restype = i32
     L.occ_ewma_update.argtypes = [vp, vp, i64, dbl, vp, vp, dbl, i32, i32, vp]
     L.occ_ewma_update.restype = i32
     L.occ_ewma_state_init.argtypes = [vp, dbl, vp]
@@ -210,6 +214,33 @@ def occ_decoupled_loss_fwd_bwd(logits, ids, logp_old, logp_mu, adv, loss_mask=No
         _ptr(dlogits), ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(),
         _stream(stream, dev))
     _check(rc, "occ_decoupled_loss_fwd_bwd")
+    return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "flags": flags_out}
+
+
+NOALLOC_MAX_TOKENS = 786432  # OCC_NOALLOC_MAX_TOKENS
+
+
+def occ_decoupled_loss_fwd_bwd_noalloc(logits, ids, logp_old, logp_mu, adv, loss_mask, *,
+                                       rd_lo, rd_hi, eps_low, eps_high, rd_weight=1,
+                                       grad_scale=1.0, denom=0, dlogits_f32=False, dlogits,
+                                       logp_out, flags_out, stats, stream=None):
+    """occ_decoupled_loss_fwd_bwd for callers that cannot allocate device memory.
+
+    Every output buffer must be supplied (``dlogits`` may be None for a
+    forward-only call); the scratch comes from the library's own fixed array,
+    so at most NOALLOC_MAX_TOKENS tokens per call, and calls must not overlap
+    on the GPU.
+    """
+    _cuda(logits, ids, logp_old, logp_mu, adv, loss_mask, dlogits, logp_out, flags_out, stats)
+    T, V, ld = _rows(logits)
+    ld_grad = dlogits.stride(0) if dlogits is not None else 0
+    p = LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
+                   float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)))
+    rc = lib().occ_decoupled_loss_fwd_bwd_noalloc(
+        _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
+        _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
+        _ptr(dlogits), ld_grad, _ptr(stats), _stream(stream, logits.device))
+    _check(rc, "occ_decoupled_loss_fwd_bwd_noalloc")
     return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "flags": flags_out}
 
 
