@@ -54,6 +54,7 @@ typedef enum { OCC_F32 = 0, OCC_BF16 = 1 } occ_dtype;
 
 /* Bits of occ_loss_stats.err (device-detected data problems). */
 #define OCC_DATA_ERR_BAD_ID 1 /* some token id was outside [0, V); those tokens were dropped */
+#define OCC_DATA_ERR_TIMEOUT 2 /* a bounded wait for an asynchronous copy gave up; outputs invalid */
 
 /* Bits of the per-token flags written by occ_decoupled_loss_fwd_bwd. */
 #define OCC_FLAG_IN_BAND 1 /* r_d inside [rd_lo, rd_hi]                        (Eq. 4) */

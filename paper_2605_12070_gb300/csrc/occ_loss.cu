@@ -23,17 +23,19 @@
 // needed by every row's gradient).  A final one-CTA kernel reduces the
 // per-token losses and flags in a fixed order (deterministic float64 loss).
 #include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <mutex>
+#include <vector>
 
 #include "occ_common.cuh"
 
 namespace occ {
 
-constexpr int kK2Threads = 512;
-constexpr int kK2Unroll = 8;
+constexpr int kK2Threads = 512;  // streaming kernel
 constexpr int kK0Threads = 1024;
 constexpr int kFinThreads = 1024;
-constexpr size_t kSliceTarget = 100 * 1024;  // two CTAs per SM
-constexpr size_t kSliceMax = 200 * 1024;     // one CTA per SM
 constexpr uint8_t kWsBadId = 0x80;           // workspace flag: dropped for a bad id
 
 struct LossKParams {
@@ -48,6 +50,8 @@ struct LossKParams {
 struct K2Args {
   const void* logits;
   int64_t T, V, ld, S, row0;
+  int64_t stage_bytes;  // shared-memory bytes of one pipeline stage (TMA kernel)
+  int* ws_err;          // device-detected error bits, OR-ed into stats.err
   const int32_t* ids;
   const float* lp_old;
   const float* lp_mu;
@@ -143,146 +147,697 @@ __device__ __forceinline__ void dropped_token_outputs(const K2Args& a, int64_t r
   if (a.flags_out) a.flags_out[row] = 0;
 }
 
-template <typename Tin, typename Tout, int NT, int U>
-__global__ void __launch_bounds__(NT, 2) k2_loss_smem(const K2Args a) {
+// Backward over one row slice held in shared memory.  dz = -g p_v (+ g at the
+// sampled token), with p_v g folded into one exponential: |dz| =
+// 2^(z L - cb) where cb = lse L - log2|g|; NEG is the sign of -g.
+template <typename Tin, typename Tout, int NT, bool NEG>
+__device__ __forceinline__ void backward_slice(const uint4* sv, int64_t nvec, int tail, float xt,
+                                               Tout* drow, float cb, float g, int64_t yl) {
   constexpr int VEC = Elem<Tin>::kVec;
-  extern __shared__ __align__(16) uint4 sm_row[];
-  __shared__ RedScratch red;
-  __shared__ __align__(16) float4 cta_part;
+#pragma unroll 4
+  for (int64_t j = threadIdx.x; j < nvec; j += NT) {
+    float x[VEC], d[VEC];
+    Elem<Tin>::unpack(sv[j], x);
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) {
+      const float e = ex2_approx(fmaf(x[q], kLog2e, -cb));
+      d[q] = NEG ? -e : e;
+    }
+    if (yl >= j * VEC && yl < (j + 1) * VEC) {
+#pragma unroll
+      for (int q = 0; q < VEC; ++q)
+        if (j * VEC + q == yl) d[q] += g;
+    }
+    OutVec<Tout, VEC>::store(drow + j * VEC, d);
+  }
+  if ((int)threadIdx.x < tail) {
+    const int64_t q = nvec * VEC + threadIdx.x;
+    const float e = ex2_approx(fmaf(xt, kLog2e, -cb));
+    float dv = NEG ? -e : e;
+    if (q == yl) dv += g;
+    out_scalar(drow + q, dv);
+  }
+}
+
+constexpr uint64_t kCopyTimeoutNs = 2000000000ull;  // a row slice lands in microseconds
+
+// Persistent, TMA-pipelined cluster kernel.  Cluster c of the grid handles rows
+// c, c + ncl, c + 2 ncl, ...; CTA `rank` of the cluster owns columns
+// [rank S, rank S + S).  Thread 0 prefetches the slice of row k + STAGES - 1
+// with one cp.async.bulk into a free shared-memory stage while the CTA works
+// on row k, so HBM reads of the next rows overlap this row's reduction,
+// cluster exchange and dlogits stores.
+template <typename Tin, typename Tout, int NT, int STAGES>
+__global__ void __launch_bounds__(NT, 2) k2_loss_tma(const K2Args a) {
+  constexpr int VEC = Elem<Tin>::kVec;
+  constexpr int NW = NT / 32;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bars[STAGES];
+  __shared__ __align__(16) float4 part[2];  // this CTA's (c, s_hi, s_lo, z_y), by valid-row parity
+  __shared__ float red_c[NW];
+  __shared__ float2 red_s[NW];
   __shared__ float bc_g, bc_cb;
 
   const uint32_t C = cluster_nctarank();
   const uint32_t rank = cluster_ctarank();
-  const int64_t row = a.row0 + blockIdx.x / C;
-  const int tid = threadIdx.x;
-  const int id = a.ids[row];
-  const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
-  const bool id_ok = (id >= 0) && ((int64_t)id < a.V);
+  const int64_t cid = blockIdx.x / C;
+  const int64_t ncl = gridDim.x / C;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int64_t T = a.T, V = a.V;
   const int64_t v0 = (int64_t)rank * a.S;
-  const int64_t n = max((int64_t)0, min(a.S, a.V - v0));
-  Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad + v0 : nullptr;
-
-  if (!(m && id_ok)) {  // uniform over the cluster: no barrier is entered
-    if (drow) zero_slice_vec<Tout, VEC, NT>(drow, n);
-    if (rank == 0 && tid == 0) dropped_token_outputs(a, row, m, id_ok);
-    return;
-  }
-
-  const Tin* zrow = (const Tin*)a.logits + row * a.ld;
-  float zy = 0.f, lpo = 0.f, lpm = 0.f, A = 0.f;
-  if (tid == 0) {
-    zy = Elem<Tin>::load(zrow + id);
-    lpo = a.lp_old[row];
-    lpm = a.lp_mu[row];
-    A = a.adv[row];
-  }
-
-  // Forward: HBM -> registers -> (shared memory copy, online log-sum-exp).
-  const uint4* zv = reinterpret_cast<const uint4*>(zrow + v0);
+  const int64_t n = max((int64_t)0, min(a.S, V - v0));
   const int64_t nvec = n / VEC;
-  LseAcc acc;
-  acc_init(acc);
-  int64_t i = tid;
-  for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
-    uint4 r[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) r[u] = ld_stream_v4(zv + i + u * NT);
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      sm_row[i + u * NT] = r[u];
-      float x[VEC];
-      Elem<Tin>::unpack(r[u], x);
-      acc_add(acc, x);
-    }
-  }
-  for (; i < nvec; i += NT) {
-    const uint4 r = ld_stream_v4(zv + i);
-    sm_row[i] = r;
-    float x[VEC];
-    Elem<Tin>::unpack(r, x);
-    acc_add(acc, x);
-  }
-  const int64_t t0 = nvec * VEC;
-  if ((int64_t)tid < n - t0) {
-    float x[1] = {Elem<Tin>::load(zrow + v0 + t0 + tid)};
-    Elem<Tin>::put(reinterpret_cast<Tin*>(sm_row) + t0 + tid, x[0]);
-    acc_add(acc, x);
-  }
+  const uint32_t bulk = (uint32_t)(nvec * 16);
+  const int tail = (int)(n - nvec * VEC);
+  const size_t stage_bytes = (size_t)a.stage_bytes;
+  const Tin* logits = (const Tin*)a.logits;
 
-  float Cr;
-  float2 Sr;
-  block_lse<NT>(acc, red, Cr, Sr);
-  if (C > 1) {
-    if (tid == 0) cta_part = make_float4(Cr, Sr.x, Sr.y, 0.f);
+  if (tid == 0) {
+    for (int st = 0; st < STAGES; ++st) mbar_init(&bars[st], 1);
+    fence_mbarrier_init();
+  }
+  __syncthreads();
+
+  auto row_ok = [&](int64_t r) -> bool {
+    const int id = a.ids[r];
+    return (a.mask == nullptr || a.mask[r] != 0) && id >= 0 && (int64_t)id < V;
+  };
+  // Producer state, thread 0 only: stages with a copy whose completion thread 0
+  // has not observed (pend), the parity each of them completes (ppar), and the
+  // parity the next copy into each stage will complete (ipar).
+  uint32_t pend = 0, ppar = 0, ipar = 0;
+  bool fault = false;
+  auto issue = [&](int64_t r, int st) {
+    const uint32_t bit = 1u << st;
+    fence_proxy_async_smem();
+    mbar_arrive_expect_tx(&bars[st], bulk);
+    tma_load_1d(smem_raw + (size_t)st * stage_bytes, logits + r * a.ld + v0, bulk, &bars[st]);
+    pend |= bit;
+    ppar = (ppar & ~bit) | (ipar & bit);
+    ipar ^= bit;
+  };
+  if (tid == 0 && bulk > 0)
+    for (int st = 0; st < STAGES - 1; ++st) {
+      const int64_t r = cid + (int64_t)st * ncl;
+      if (r < T && row_ok(r)) issue(r, st);
+    }
+
+  const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
+  uint32_t phase = 0;  // consumer side: parity of the next completion of each stage
+  int64_t nvalid_done = 0;
+  int k = 0;
+  for (int64_t row = cid; row < T; row += ncl, ++k) {
+    const int st = k % STAGES;
+    if (tid == 0 && bulk > 0 && !fault) {
+      const int64_t r = row + (int64_t)(STAGES - 1) * ncl;
+      const int sn = (k + STAGES - 1) % STAGES;
+      if (r < T && row_ok(r)) issue(r, sn);
+    }
+    const int id = a.ids[row];
+    const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
+    const bool id_ok = id >= 0 && (int64_t)id < V;
+    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad + v0 : nullptr;
+    if (!(m && id_ok)) {  // uniform over the cluster: no barrier is entered
+      if (drow) zero_slice_vec<Tout, VEC, NT>(drow, n);
+      if (rank == 0 && tid == 0) dropped_token_outputs(a, row, m, id_ok);
+      continue;
+    }
+    float lpo = 0.f, lpm = 0.f, A = 0.f;
+    if (tid == 0) {
+      lpo = a.lp_old[row];
+      lpm = a.lp_mu[row];
+      A = a.adv[row];
+    }
+    unsigned char* sp = smem_raw + (size_t)st * stage_bytes;
+    if (bulk > 0) {
+      const uint32_t par = (phase >> st) & 1u;
+      const bool ok = mbar_wait_bounded(&bars[st], par, fault ? 0 : kCopyTimeoutNs);
+      phase ^= 1u << st;
+      if (!ok) fault = true;
+      if (tid == 0 && ok) pend &= ~(1u << st);
+    }
+    // ragged tail of the last slice: plain loads, kept in registers and smem
+    const Tin* zs = logits + row * a.ld + v0;
+    float xt = 0.f;
+    LseAcc acc;
+    acc_init(acc);
+    if (tid < tail) {
+      xt = Elem<Tin>::load(zs + nvec * VEC + tid);
+      Elem<Tin>::put(reinterpret_cast<Tin*>(sp) + nvec * VEC + tid, xt);
+      float x1[1] = {xt};
+      acc_add(acc, x1);
+    }
+    // forward: online log-sum-exp over the slice in shared memory
+    const uint4* sv = reinterpret_cast<const uint4*>(sp);
+#pragma unroll 4
+    for (int64_t j = tid; j < nvec; j += NT) {
+      float x[VEC];
+      Elem<Tin>::unpack(sv[j], x);
+      acc_add_fast(acc, x);
+    }
+    // CTA reduction: warp max, one rescale per lane, compensated warp sums
+    const float wmax = warp_max(acc.c);
+    float2 v = make_float2(acc.c == -INFINITY ? 0.f : acc.s * exp2f(acc.c - wmax), 0.f);
+    v = warp_pair_sum(v);
+    if (lane == 0) {
+      red_c[wid] = wmax;
+      red_s[wid] = v;
+    }
+    __syncthreads();
+    const int slot = (int)(nvalid_done & 1);
+    if (wid == 0) {
+      const float c = lane < NW ? red_c[lane] : -INFINITY;
+      const float cm = warp_max(c);
+      float2 w = make_float2(0.f, 0.f);
+      if (lane < NW && c != -INFINITY) {
+        const float f = exp2f(c - cm);
+        const float2 p = red_s[lane];
+        const float hi = p.x * f;
+        w = make_float2(hi, fmaf(p.x, f, -hi) + p.y * f);
+      }
+      w = warp_pair_sum(w);
+      if (lane == 0) {
+        const int64_t yl = (int64_t)id - v0;
+        float zy = 0.f;
+        if (yl >= 0 && yl < n) {
+          if (sizeof(Tin) == 2)
+            zy = __uint_as_float(((uint32_t)reinterpret_cast<const uint16_t*>(sp)[yl]) << 16);
+          else
+            zy = reinterpret_cast<const float*>(sp)[yl];
+        }
+        part[slot] = make_float4(cm, w.x, w.y, zy);
+      }
+    }
+    // exchange the C partials (cluster barrier; a CTA barrier when C = 1)
+    if (C > 1) {
+      cluster_arrive_release();
+      cluster_wait_acquire();
+    } else {
+      __syncthreads();
+    }
+    if (wid == 0) {
+      float4 P = make_float4(-INFINITY, 0.f, 0.f, 0.f);
+      if (lane < (int)C) P = (C > 1) ? ld_dsmem_f4(&part[slot], (uint32_t)lane) : part[slot];
+      const float cm = warp_max(P.x);
+      float2 w = make_float2(0.f, 0.f);
+      if (lane < (int)C && P.x != -INFINITY) {
+        const float f = exp2f(P.x - cm);
+        const float hi = P.y * f;
+        w = make_float2(hi, fmaf(P.y, f, -hi) + P.z * f);
+      }
+      w = warp_pair_sum(w);
+      const float zy = __shfl_sync(0xffffffffu, P.w, (int)((int64_t)id / a.S));
+      if (lane == 0) {
+        const double lse = lse_from(cm, w);
+        float g, loss_t, logp_f;
+        uint32_t fl;
+        token_math(a.kp, lse, zy, lpo, lpm, A, N, g, loss_t, fl, logp_f);
+        float cb = 0.f;
+        if (g != 0.f) {
+          int e;
+          const float fm = frexpf(fabsf(g), &e);  // |g| = fm 2^e
+          cb = (float)(lse * (double)kLog2e - (double)e - (double)log2f(fm));
+        }
+        bc_g = g;
+        bc_cb = cb;
+        if (rank == 0) {
+          a.ws_loss[row] = loss_t;
+          a.ws_flags[row] = (uint8_t)fl;
+          if (a.logp_out) a.logp_out[row] = logp_f;
+          if (a.flags_out) a.flags_out[row] = (uint8_t)fl;
+        }
+      }
+    }
+    __syncthreads();
+    if (drow) {
+      const float g = bc_g;
+      if (g == 0.f) {
+        zero_slice_vec<Tout, VEC, NT>(drow, n);
+      } else if (g > 0.f) {
+        backward_slice<Tin, Tout, NT, true>(sv, nvec, tail, xt, drow, bc_cb, g, (int64_t)id - v0);
+      } else {
+        backward_slice<Tin, Tout, NT, false>(sv, nvec, tail, xt, drow, bc_cb, g, (int64_t)id - v0);
+      }
+    }
+    __syncthreads();  // stage st and the broadcast slots are free again
+    ++nvalid_done;
+  }
+  if (C > 1) {  // no CTA leaves while a peer may still read its partials
     cluster_arrive_release();
     cluster_wait_acquire();
-    if (tid == 0) {  // merge the C partials in rank order (same order in every CTA)
-      float Cm = -INFINITY;
-      for (uint32_t r = 0; r < C; ++r) Cm = fmaxf(Cm, ld_dsmem_f4(&cta_part, r).x);
-      float2 s = make_float2(0.f, 0.f);
-      for (uint32_t r = 0; r < C; ++r) {
-        const float4 P = ld_dsmem_f4(&cta_part, r);
-        if (P.x == -INFINITY) continue;
-        const float f = exp2f(P.x - Cm);
-        const float hi = P.y * f;
-        s = pair_add(s, make_float2(hi, fmaf(P.y, f, -hi) + P.z * f));
-      }
-      Cr = Cm;
-      Sr = s;
-    }
-    cluster_arrive_release();  // this CTA is done reading the others' shared memory
   }
+  if (tid == 0) {
+    if (fault) atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
+    // copies still in flight (only after a timeout): wait, bounded, before exiting
+    for (int st = 0; st < STAGES; ++st)
+      if (pend & (1u << st)) {
+        if (!mbar_wait_bounded(&bars[st], (ppar >> st) & 1u, kCopyTimeoutNs))
+          atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
+      }
+  }
+}
+
+// Packed bf16 max of the eight values of a 16-byte vector, as a float.
+__device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+template <typename Tin>
+struct VecMax;
+template <>
+struct VecMax<bf16_t> {
+  __device__ __forceinline__ static float of(const uint4& r) {
+    const uint32_t m = bf16x2_max(bf16x2_max(r.x, r.y), bf16x2_max(r.z, r.w));
+    return fmaxf(bf16_lo(m), bf16_hi(m));
+  }
+};
+template <>
+struct VecMax<float> {
+  __device__ __forceinline__ static float of(const uint4& r) {
+    return fmaxf(fmaxf(__uint_as_float(r.x), __uint_as_float(r.y)),
+                 fmaxf(__uint_as_float(r.z), __uint_as_float(r.w)));
+  }
+};
+
+// Register-resident persistent kernel for rows whose CTA slice fits EV
+// vectors per thread.  The forward pass keeps every term e_v = 2^(z_v L - c)
+// of the thread's share of the slice in registers (c = the thread's own
+// maximum, so e_v <= 1), which makes the backward a multiplication:
+//   dz_v = k e_v (+ g at the sampled token),  k = -g 2^(c - lse L),
+// one exponential per element for forward and backward together.  The
+// shared-memory stage only lands the TMA copy and is handed back to the
+// prefetcher as soon as the forward pass has read it.
+template <typename Tin, typename Tout, int NT, int EV, int STAGES>
+__global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
+  constexpr int VEC = Elem<Tin>::kVec;
+  constexpr int NW = NT / 32;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bars[STAGES];
+  __shared__ __align__(16) float4 part[2];  // (c, s_hi, s_lo, z_y) by valid-row parity
+  __shared__ float red_c[NW];
+  __shared__ float2 red_s[NW];
+  __shared__ float bc_g, zy_sh;
+  __shared__ double bc_lseL;
+
+  const uint32_t C = cluster_nctarank();
+  const uint32_t rank = cluster_ctarank();
+  const int64_t cid = blockIdx.x / C;
+  const int64_t ncl = gridDim.x / C;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int64_t T = a.T, V = a.V;
+  const int64_t v0 = (int64_t)rank * a.S;
+  const int64_t n = max((int64_t)0, min(a.S, V - v0));
+  const int64_t nvec = n / VEC;
+  const uint32_t bulk = (uint32_t)(nvec * 16);
+  const int tail = (int)(n - nvec * VEC);
+  const size_t stage_bytes = (size_t)a.stage_bytes;
+  const Tin* logits = (const Tin*)a.logits;
 
   if (tid == 0) {
-    const double lse = lse_from(Cr, Sr);
-    const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
-    float g, loss_t, logp_f;
-    uint32_t fl;
-    token_math(a.kp, lse, zy, lpo, lpm, A, N, g, loss_t, fl, logp_f);
-    bc_g = g;
-    bc_cb = (float)(lse * (double)kLog2e);  // p_v = 2^(z_v L - cb)
-    if (rank == 0) {
+    for (int st = 0; st < STAGES; ++st) mbar_init(&bars[st], 1);
+    fence_mbarrier_init();
+  }
+  __syncthreads();
+
+  auto row_ok = [&](int64_t r) -> bool {
+    const int id = a.ids[r];
+    return (a.mask == nullptr || a.mask[r] != 0) && id >= 0 && (int64_t)id < V;
+  };
+  uint32_t pend = 0, ppar = 0, ipar = 0;  // producer bookkeeping (thread 0)
+  bool fault = false;
+  auto issue = [&](int64_t r, int st) {
+    const uint32_t bit = 1u << st;
+    fence_proxy_async_smem();
+    mbar_arrive_expect_tx(&bars[st], bulk);
+    tma_load_1d(smem_raw + (size_t)st * stage_bytes, logits + r * a.ld + v0, bulk, &bars[st]);
+    pend |= bit;
+    ppar = (ppar & ~bit) | (ipar & bit);
+    ipar ^= bit;
+  };
+  // refill stage st with the row STAGES iterations ahead (thread 0)
+  auto refill = [&](int64_t row, int st) {
+    if (tid == 0 && bulk > 0 && !fault) {
+      const int64_t r = row + (int64_t)STAGES * ncl;
+      if (r < T && row_ok(r)) issue(r, st);
+    }
+  };
+  if (tid == 0 && bulk > 0)
+    for (int st = 0; st < STAGES; ++st) {
+      const int64_t r = cid + (int64_t)st * ncl;
+      if (r < T && row_ok(r)) issue(r, st);
+    }
+
+  const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
+  uint32_t phase = 0;
+  int64_t nvalid_done = 0;
+  int k = 0;
+  for (int64_t row = cid; row < T; row += ncl, ++k) {
+    const int st = k % STAGES;
+    const int id = a.ids[row];
+    const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
+    const bool id_ok = id >= 0 && (int64_t)id < V;
+    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad + v0 : nullptr;
+    if (!(m && id_ok)) {  // uniform over the cluster: no barrier is entered
+      refill(row, st);
+      if (drow) zero_slice_vec<Tout, VEC, NT>(drow, n);
+      if (rank == 0 && tid == 0) dropped_token_outputs(a, row, m, id_ok);
+      continue;
+    }
+    float lpo = 0.f, lpm = 0.f, A = 0.f;
+    if (tid == 0) {
+      lpo = a.lp_old[row];
+      lpm = a.lp_mu[row];
+      A = a.adv[row];
+    }
+    const unsigned char* sp = smem_raw + (size_t)st * stage_bytes;
+    if (bulk > 0) {
+      const bool ok = mbar_wait_bounded(&bars[st], (phase >> st) & 1u, fault ? 0 : kCopyTimeoutNs);
+      phase ^= 1u << st;
+      if (!ok) fault = true;
+      if (tid == 0 && ok) pend &= ~(1u << st);
+    }
+    const int64_t yl = (int64_t)id - v0;  // sampled token in slice coordinates
+    float xt = -INFINITY;
+    if (tid < tail) xt = Elem<Tin>::load(logits + row * a.ld + v0 + nvec * VEC + tid);
+    // pass 1: the thread's maximum
+    const uint4* sv = reinterpret_cast<const uint4*>(sp);
+    float mx = xt;
+#pragma unroll
+    for (int e = 0; e < EV; ++e) {
+      const int64_t j = tid + (int64_t)e * NT;
+      if (j < nvec) mx = fmaxf(mx, VecMax<Tin>::of(sv[j]));
+    }
+    const float c = mx * kLog2e;  // -inf when the thread holds nothing finite
+    // pass 2: terms e_v = 2^(z_v L - c) kept in registers
+    float E[EV][VEC];
+    float s = 0.f, et = 0.f;
+    if (c != -INFINITY) {
+#pragma unroll
+      for (int e = 0; e < EV; ++e) {
+        const int64_t j = tid + (int64_t)e * NT;
+        if (j < nvec) {
+          float x[VEC];
+          Elem<Tin>::unpack(sv[j], x);
+          float t = 0.f;
+#pragma unroll
+          for (int q = 0; q < VEC; ++q) {
+            E[e][q] = ex2_approx(fmaf(x[q], kLog2e, -c));
+            t += E[e][q];
+          }
+          s += t;
+          if (yl >= j * VEC && yl < (j + 1) * VEC) {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q)
+              if (j * VEC + q == yl) zy_sh = x[q];
+          }
+        }
+      }
+      if (tid < tail) {
+        et = ex2_approx(fmaf(xt, kLog2e, -c));
+        s += et;
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < EV; ++e)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) E[e][q] = 0.f;
+    }
+    if (tid < tail && nvec * VEC + tid == yl) zy_sh = xt;
+    // CTA reduction: warp max, one rescale per lane, compensated warp sums
+    const float wmax = warp_max(c);
+    float2 v = make_float2(c == -INFINITY ? 0.f : s * exp2f(c - wmax), 0.f);
+    v = warp_pair_sum(v);
+    if (lane == 0) {
+      red_c[wid] = wmax;
+      red_s[wid] = v;
+    }
+    __syncthreads();   // the stage has been read: hand it to the prefetcher
+    refill(row, st);
+    const int slot = (int)(nvalid_done & 1);
+    if (wid == 0) {
+      const float cw = lane < NW ? red_c[lane] : -INFINITY;
+      const float cm = warp_max(cw);
+      float2 w = make_float2(0.f, 0.f);
+      if (lane < NW && cw != -INFINITY) {
+        const float f = exp2f(cw - cm);
+        const float2 p = red_s[lane];
+        const float hi = p.x * f;
+        w = make_float2(hi, fmaf(p.x, f, -hi) + p.y * f);
+      }
+      w = warp_pair_sum(w);
+      if (lane == 0) part[slot] = make_float4(cm, w.x, w.y, (yl >= 0 && yl < n) ? zy_sh : 0.f);
+    }
+    if (C > 1) {
+      cluster_arrive_release();
+      cluster_wait_acquire();
+    } else {
+      __syncthreads();
+    }
+    if (wid == 0) {
+      float4 P = make_float4(-INFINITY, 0.f, 0.f, 0.f);
+      if (lane < (int)C) P = (C > 1) ? ld_dsmem_f4(&part[slot], (uint32_t)lane) : part[slot];
+      const float cm = warp_max(P.x);
+      float2 w = make_float2(0.f, 0.f);
+      if (lane < (int)C && P.x != -INFINITY) {
+        const float f = exp2f(P.x - cm);
+        const float hi = P.y * f;
+        w = make_float2(hi, fmaf(P.y, f, -hi) + P.z * f);
+      }
+      w = warp_pair_sum(w);
+      const float zy = __shfl_sync(0xffffffffu, P.w, (int)((int64_t)id / a.S));
+      if (lane == 0) {
+        const double lse = lse_from(cm, w);
+        float g, loss_t, logp_f;
+        uint32_t fl;
+        token_math(a.kp, lse, zy, lpo, lpm, A, N, g, loss_t, fl, logp_f);
+        bc_g = g;
+        bc_lseL = lse * (double)kLog2e;
+        if (rank == 0) {
+          a.ws_loss[row] = loss_t;
+          a.ws_flags[row] = (uint8_t)fl;
+          if (a.logp_out) a.logp_out[row] = logp_f;
+          if (a.flags_out) a.flags_out[row] = (uint8_t)fl;
+        }
+      }
+    }
+    __syncthreads();
+    if (drow) {
+      const float g = bc_g;
+      if (g == 0.f) {
+        zero_slice_vec<Tout, VEC, NT>(drow, n);
+      } else {
+        const float kf = c == -INFINITY ? 0.f : -g * exp2f((float)((double)c - bc_lseL));
+#pragma unroll
+        for (int e = 0; e < EV; ++e) {
+          const int64_t j = tid + (int64_t)e * NT;
+          if (j < nvec) {
+            float d[VEC];
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) d[q] = kf * E[e][q];
+            if (yl >= j * VEC && yl < (j + 1) * VEC) {
+#pragma unroll
+              for (int q = 0; q < VEC; ++q)
+                if (j * VEC + q == yl) d[q] += g;
+            }
+            OutVec<Tout, VEC>::store(drow + j * VEC, d);
+          }
+        }
+        if (tid < tail) {
+          const int64_t q = nvec * VEC + tid;
+          float dv = kf * et;
+          if (q == yl) dv += g;
+          out_scalar(drow + q, dv);
+        }
+      }
+    }
+    ++nvalid_done;
+  }
+  if (C > 1) {  // no CTA leaves while a peer may still read its partials
+    cluster_arrive_release();
+    cluster_wait_acquire();
+  }
+  if (tid == 0) {
+    if (fault) atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
+    for (int st = 0; st < STAGES; ++st)
+      if (pend & (1u << st)) {
+        if (!mbar_wait_bounded(&bars[st], (ppar >> st) & 1u, kCopyTimeoutNs))
+          atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
+      }
+  }
+}
+
+// Writes VEC gradient values with an L2 policy (16 bytes per 8 bf16 / 4 f32).
+template <typename Tout, int VEC>
+struct OutVecHint;
+template <>
+struct OutVecHint<bf16_t, 8> {
+  __device__ __forceinline__ static void store(bf16_t* p, const float (&d)[8], uint64_t pol) {
+    st_hint_v4(p, make_uint4(pack_bf16x2(d[0], d[1]), pack_bf16x2(d[2], d[3]),
+                             pack_bf16x2(d[4], d[5]), pack_bf16x2(d[6], d[7])), pol);
+  }
+  __device__ __forceinline__ static void zero(bf16_t* p, uint64_t pol) {
+    st_hint_v4(p, make_uint4(0, 0, 0, 0), pol);
+  }
+};
+template <>
+struct OutVecHint<float, 8> {
+  __device__ __forceinline__ static void store(float* p, const float (&d)[8], uint64_t pol) {
+    st_hint_v4(p, make_uint4(__float_as_uint(d[0]), __float_as_uint(d[1]), __float_as_uint(d[2]),
+                             __float_as_uint(d[3])), pol);
+    st_hint_v4(p + 4, make_uint4(__float_as_uint(d[4]), __float_as_uint(d[5]),
+                                 __float_as_uint(d[6]), __float_as_uint(d[7])), pol);
+  }
+  __device__ __forceinline__ static void zero(float* p, uint64_t pol) {
+    st_hint_v4(p, make_uint4(0, 0, 0, 0), pol);
+    st_hint_v4(p + 4, make_uint4(0, 0, 0, 0), pol);
+  }
+};
+template <>
+struct OutVecHint<float, 4> {
+  __device__ __forceinline__ static void store(float* p, const float (&d)[4], uint64_t pol) {
+    st_hint_v4(p, make_uint4(__float_as_uint(d[0]), __float_as_uint(d[1]), __float_as_uint(d[2]),
+                             __float_as_uint(d[3])), pol);
+  }
+  __device__ __forceinline__ static void zero(float* p, uint64_t pol) {
+    st_hint_v4(p, make_uint4(0, 0, 0, 0), pol);
+  }
+};
+
+// One CTA per row, two streaming passes (the K1 layout).  The forward pass
+// reads the row from HBM with an L2 evict-last policy; the backward pass
+// re-reads it with evict-first (its last use), so with one or two rows in
+// flight per SM the re-read is served by the 129 MB L2 and HBM sees the
+// logits once and dlogits once.  dlogits are written evict-first.
+template <typename Tin, typename Tout, int NT, int U>
+__global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
+  constexpr int VEC = Elem<Tin>::kVec;
+  __shared__ RedScratch red;
+  __shared__ float bc_g, bc_cb;
+  const uint64_t keep = l2_policy_evict_last();
+  const uint64_t last = l2_policy_evict_first();
+  const int tid = threadIdx.x;
+  const int64_t V = a.V;
+  const int64_t nvec = V / VEC;
+  const int64_t tail0 = nvec * VEC;
+  const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
+  for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
+    const int id = a.ids[row];
+    const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
+    const bool id_ok = id >= 0 && (int64_t)id < V;
+    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    if (!(m && id_ok)) {
+      if (drow) {
+        for (int64_t i = tid; i < nvec; i += NT) OutVecHint<Tout, VEC>::zero(drow + i * VEC, last);
+        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+      }
+      if (tid == 0) dropped_token_outputs(a, row, m, id_ok);
+      continue;
+    }
+    const Tin* z = (const Tin*)a.logits + row * a.ld;
+    float zy = 0.f, lpo = 0.f, lpm = 0.f, A = 0.f;
+    if (tid == 0) {
+      zy = Elem<Tin>::load(z + id);
+      lpo = a.lp_old[row];
+      lpm = a.lp_mu[row];
+      A = a.adv[row];
+    }
+    const uint4* zv = reinterpret_cast<const uint4*>(z);
+    LseAcc acc;
+    acc_init(acc);
+    int64_t i = tid;
+    for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
+      uint4 r[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + i + u * NT, keep);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        float x[VEC];
+        Elem<Tin>::unpack(r[u], x);
+        acc_add_fast(acc, x);
+      }
+    }
+    for (; i < nvec; i += NT) {
+      float x[VEC];
+      Elem<Tin>::unpack(ld_hint_v4(zv + i, keep), x);
+      acc_add_fast(acc, x);
+    }
+    float xt = 0.f;
+    if ((int64_t)tid < V - tail0) {
+      xt = Elem<Tin>::load(z + tail0 + tid);
+      float x1[1] = {xt};
+      acc_add(acc, x1);
+    }
+    float Cr;
+    float2 Sr;
+    block_lse<NT>(acc, red, Cr, Sr);
+    if (tid == 0) {
+      const double lse = lse_from(Cr, Sr);
+      float g, loss_t, logp_f;
+      uint32_t fl;
+      token_math(a.kp, lse, zy, lpo, lpm, A, N, g, loss_t, fl, logp_f);
+      float cb = 0.f;
+      if (g != 0.f) {
+        int e;
+        const float fm = frexpf(fabsf(g), &e);
+        cb = (float)(lse * (double)kLog2e - (double)e - (double)log2f(fm));
+      }
+      bc_g = g;
+      bc_cb = cb;
       a.ws_loss[row] = loss_t;
       a.ws_flags[row] = (uint8_t)fl;
       if (a.logp_out) a.logp_out[row] = logp_f;
       if (a.flags_out) a.flags_out[row] = (uint8_t)fl;
     }
-  }
-  __syncthreads();
-
-  // Backward straight from shared memory.
-  if (drow) {
-    const float g = bc_g;
-    if (g == 0.f) {
-      zero_slice_vec<Tout, VEC, NT>(drow, n);
-    } else {
-      const float cb = bc_cb;
-      const int64_t yl = (int64_t)id - v0;  // sampled token, local index (may be outside)
-#pragma unroll 4
-      for (int64_t j = tid; j < nvec; j += NT) {
-        float x[VEC], d[VEC];
-        Elem<Tin>::unpack(sm_row[j], x);
+    __syncthreads();
+    if (drow) {
+      const float g = bc_g, cb = bc_cb;
+      if (g == 0.f) {
+        for (int64_t j = tid; j < nvec; j += NT) OutVecHint<Tout, VEC>::zero(drow + j * VEC, last);
+        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+      } else {
+        const float sgn = g > 0.f ? -1.f : 1.f;
+        int64_t j = tid;
+        for (; j + (int64_t)(U - 1) * NT < nvec; j += (int64_t)U * NT) {
+          uint4 r[U];
 #pragma unroll
-        for (int k = 0; k < VEC; ++k) {
-          d[k] = -g * ex2_approx(fmaf(x[k], kLog2e, -cb));
-          if (j * VEC + k == yl) d[k] += g;
+          for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + j + u * NT, last);
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int64_t jj = j + u * NT;
+            float x[VEC], d[VEC];
+            Elem<Tin>::unpack(r[u], x);
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
+            if (id >= jj * VEC && id < (jj + 1) * VEC) {
+#pragma unroll
+              for (int q = 0; q < VEC; ++q)
+                if (jj * VEC + q == id) d[q] += g;
+            }
+            OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
+          }
         }
-        OutVec<Tout, VEC>::store(drow + j * VEC, d);
-      }
-      if ((int64_t)tid < n - t0) {
-        const int64_t k = t0 + tid;
-        float xs;
-        if (sizeof(Tin) == 2)
-          xs = __uint_as_float(((uint32_t)reinterpret_cast<const uint16_t*>(sm_row)[k]) << 16);
-        else
-          xs = reinterpret_cast<const float*>(sm_row)[k];
-        float dv = -g * ex2_approx(fmaf(xs, kLog2e, -cb));
-        if (k == yl) dv += g;
-        out_scalar(drow + k, dv);
+        for (; j < nvec; j += NT) {
+          float x[VEC], d[VEC];
+          Elem<Tin>::unpack(ld_hint_v4(zv + j, last), x);
+#pragma unroll
+          for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
+          if (id >= j * VEC && id < (j + 1) * VEC) {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q)
+              if (j * VEC + q == id) d[q] += g;
+          }
+          OutVecHint<Tout, VEC>::store(drow + j * VEC, d, last);
+        }
+        if ((int64_t)tid < V - tail0) {
+          float dv = sgn * ex2_approx(fmaf(xt, kLog2e, -cb));
+          if (tail0 + tid == id) dv += g;
+          out_scalar(drow + tail0 + tid, dv);
+        }
       }
     }
+    __syncthreads();
   }
-  if (C > 1) cluster_wait_acquire();
 }
 
 // Any alignment / any V: element loads, forward pass then backward pass over
@@ -357,8 +912,10 @@ __global__ void __launch_bounds__(NT) k2_loss_stream(const K2Args a) {
 template <int NT>
 __global__ void __launch_bounds__(NT) k0_count_valid(const uint8_t* __restrict__ mask,
                                                      const int32_t* __restrict__ ids, int64_t T,
-                                                     int64_t V, long long* __restrict__ ws_N) {
+                                                     int64_t V, long long* __restrict__ ws_N,
+                                                     int* __restrict__ ws_err) {
   __shared__ long long part[NT / 32];
+  if (threadIdx.x == 0) *ws_err = 0;
   long long c = 0;
   for (int64_t t0 = threadIdx.x; t0 < T; t0 += 8 * (int64_t)NT) {
     int idv[8];
@@ -388,6 +945,7 @@ template <int NT>
 __global__ void __launch_bounds__(NT) k2_finalize(int64_t T, const float* __restrict__ ws_loss,
                                                   const uint8_t* __restrict__ ws_flags,
                                                   const long long* __restrict__ ws_N,
+                                                  const int* __restrict__ ws_err,
                                                   long long denom_fixed, occ_loss_stats* st) {
   __shared__ float2 ps[NT / 32];
   __shared__ long long pc[4][NT / 32];
@@ -444,7 +1002,7 @@ __global__ void __launch_bounds__(NT) k2_finalize(int64_t T, const float* __rest
     st->n_clipped = c[2];
     st->n_active = c[3];
     st->denom = N;
-    st->err = b ? OCC_DATA_ERR_BAD_ID : 0;
+    st->err = (b ? OCC_DATA_ERR_BAD_ID : 0) | *ws_err;
     st->reserved = 0;
   }
 }
@@ -454,12 +1012,13 @@ __global__ void __launch_bounds__(NT) k2_finalize(int64_t T, const float* __rest
 static inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct WsLayout {
-  size_t off_N, off_loss, off_flags, total;
+  size_t off_N, off_err, off_loss, off_flags, total;
 };
 static WsLayout ws_layout(int64_t T) {
   const size_t t = T > 0 ? (size_t)T : 0;
   WsLayout w;
   w.off_N = 0;
+  w.off_err = 8;
   w.off_loss = 256;
   w.off_flags = w.off_loss + align_up(4 * t, 256);
   w.total = w.off_flags + align_up(t, 256);
@@ -467,64 +1026,175 @@ static WsLayout ws_layout(int64_t T) {
 }
 
 struct ClusterPlan {
-  int C;       // CTAs per row (0: use the streaming kernel)
-  int64_t S;   // elements per CTA slice (multiple of the vector width)
-  size_t smem; // dynamic shared memory per CTA
+  int C;               // CTAs per row (0: use the streaming kernel)
+  int64_t S;           // elements per CTA slice (multiple of the vector width)
+  size_t stage_bytes;  // one pipeline stage, rounded to 128 bytes
 };
 
-static ClusterPlan plan_cluster(int64_t V, size_t es) {
+constexpr int kK2Stages = 2;
+constexpr size_t kSmemTarget = 80 * 1024;   // two CTAs per SM
+constexpr size_t kSmemMax = 200 * 1024;     // one CTA per SM
+
+static ClusterPlan plan_cluster(int64_t V, size_t es, int stages) {
   const int64_t vec = 16 / (int64_t)es;
-  for (size_t cap : {kSliceTarget, kSliceMax}) {
+  for (size_t cap : {kSmemTarget, kSmemMax}) {
     for (int C : {1, 2, 4, 8}) {
       int64_t S = (V + C - 1) / C;
       S = (S + vec - 1) / vec * vec;
-      if ((size_t)S * es <= cap) return ClusterPlan{C, S, (size_t)S * es};
+      const size_t sb = align_up((size_t)S * es, 128);
+      if (sb * stages <= cap) return ClusterPlan{C, S, sb};
     }
   }
   return ClusterPlan{0, V, 0};
 }
 
+// Co-resident clusters for a kernel configuration (cached per device).
+static int max_active_clusters(const void* kern, int C, int NT, size_t smem) {
+  struct Key {
+    const void* k;
+    int C, NT, dev;
+    size_t smem;
+    int n;
+  };
+  static std::mutex mu;
+  static std::vector<Key> cache;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lk(mu);
+  for (const Key& e : cache)
+    if (e.k == kern && e.C == C && e.NT == NT && e.dev == dev && e.smem == smem) return e.n;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(C, 1, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  cache.push_back(Key{kern, C, NT, dev, smem, n});
+  return n;
+}
+
+template <typename Kern>
+static occ_status launch_persistent(Kern kern, int NT, K2Args a, const ClusterPlan& pl, int stages,
+                                    cudaStream_t s) {
+  const size_t smem = (size_t)stages * pl.stage_bytes;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess)
+    return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", smem, cudaGetErrorString(e));
+  int ncl = max_active_clusters((const void*)kern, pl.C, NT, smem);
+  if (ncl <= 0)
+    return fail(OCC_ERR_CUDA, "no co-resident cluster of %d CTAs with %zu bytes of shared memory",
+                pl.C, smem);
+  ncl = (int)std::min<int64_t>(ncl, a.T);
+  a.S = pl.S;
+  a.stage_bytes = (int64_t)pl.stage_bytes;
+  a.row0 = 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(ncl * pl.C), 1, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = pl.C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, a);
+  if (e != cudaSuccess)
+    return fail(OCC_ERR_CUDA, "k2 launch (clusters=%d x %d CTAs, smem=%zu): %s", ncl, pl.C, smem,
+                cudaGetErrorString(e));
+  return check_launch("occ_decoupled_loss_fwd_bwd");
+}
+
+// Register-resident kernel geometry: 256 threads, 80 float registers of terms
+// per thread, so a CTA slice holds at most 20480 elements.
+constexpr int kRegThreads = 256;
+constexpr int64_t kRegSliceElems = 20480;
+
+static ClusterPlan plan_reg(int64_t V, size_t es, int stages) {
+  const int64_t vec = 16 / (int64_t)es;
+  for (int C : {1, 2, 4, 8}) {
+    int64_t S = (V + C - 1) / C;
+    S = (S + vec - 1) / vec * vec;
+    const size_t sb = align_up((size_t)S * es, 128);
+    if (S <= kRegSliceElems && sb * stages <= kSmemMax) return ClusterPlan{C, S, sb};
+  }
+  return ClusterPlan{0, V, 0};
+}
+
+// Threads per CTA of the TMA kernel (OCC_K2_THREADS=256|512 overrides, for tuning).
+static int k2_threads() {
+  static int nt = [] {
+    const char* v = getenv("OCC_K2_THREADS");
+    return (v && atoi(v) == 512) ? 512 : 256;
+  }();
+  return nt;
+}
+
+// Kernel variant for aligned rows: "l2" (default), "reg" or "tma"
+// (OCC_K2_VARIANT overrides, for tuning).
+static int k2_variant() {
+  static int v = [] {
+    const char* e = getenv("OCC_K2_VARIANT");
+    if (e && !strcmp(e, "reg")) return 1;
+    if (e && !strcmp(e, "tma")) return 2;
+    if (e && !strcmp(e, "l2_1024")) return 3;
+    return 0;
+  }();
+  return v;
+}
+
 template <typename Tin, typename Tout>
 static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
   const int64_t T = a.T;
-  ClusterPlan pl = vec ? plan_cluster(a.V, sizeof(Tin)) : ClusterPlan{0, a.V, 0};
-  if (pl.C == 0) {
+  if (vec) {
+    const int var = k2_variant();
+    if (var == 1) {
+      const ClusterPlan pr = plan_reg(a.V, sizeof(Tin), kK2Stages);
+      if (pr.C > 0) {
+        constexpr int EV = (int)(kRegSliceElems / kRegThreads / Elem<Tin>::kVec);
+        return launch_persistent(k2_loss_reg<Tin, Tout, kRegThreads, EV, kK2Stages>, kRegThreads,
+                                 a, pr, kK2Stages, s);
+      }
+    }
+    if (var == 2) {
+      const ClusterPlan pl = plan_cluster(a.V, sizeof(Tin), kK2Stages);
+      if (pl.C > 0) {
+        if (k2_threads() == 512)
+          return launch_persistent(k2_loss_tma<Tin, Tout, 512, kK2Stages>, 512, a, pl, kK2Stages,
+                                   s);
+        return launch_persistent(k2_loss_tma<Tin, Tout, 256, kK2Stages>, 256, a, pl, kK2Stages, s);
+      }
+    }
     const int64_t step = 0x7fffffffLL;
     for (int64_t r0 = 0; r0 < T; r0 += step) {
       a.row0 = r0;
       const unsigned grid = (unsigned)std::min<int64_t>(step, T - r0);
-      k2_loss_stream<Tin, Tout, kK2Threads><<<grid, kK2Threads, 0, s>>>(a);
+      if (var == 3)
+        k2_loss_l2<Tin, Tout, 1024, 8><<<grid, 1024, 0, s>>>(a);
+      else
+        k2_loss_l2<Tin, Tout, 512, 8><<<grid, 512, 0, s>>>(a);
     }
-    return check_launch("occ_decoupled_loss_fwd_bwd (stream kernel)");
+    return check_launch("occ_decoupled_loss_fwd_bwd");
   }
-  auto kern = k2_loss_smem<Tin, Tout, kK2Threads, kK2Unroll>;
-  cudaError_t e =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem);
-  if (e != cudaSuccess)
-    return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", pl.smem, cudaGetErrorString(e));
-  a.S = pl.S;
-  const int64_t step = 0x7fffffffLL / pl.C;
+  const int64_t step = 0x7fffffffLL;
   for (int64_t r0 = 0; r0 < T; r0 += step) {
     a.row0 = r0;
-    const int64_t rows = std::min<int64_t>(step, T - r0);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(rows * pl.C), 1, 1);
-    cfg.blockDim = dim3(kK2Threads, 1, 1);
-    cfg.dynamicSmemBytes = pl.smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = pl.C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = pl.C > 1 ? 1 : 0;
-    e = cudaLaunchKernelEx(&cfg, kern, a);
-    if (e != cudaSuccess)
-      return fail(OCC_ERR_CUDA, "k2 cluster launch (C=%d, smem=%zu): %s", pl.C, pl.smem,
-                  cudaGetErrorString(e));
+    const unsigned grid = (unsigned)std::min<int64_t>(step, T - r0);
+    k2_loss_stream<Tin, Tout, kK2Threads><<<grid, kK2Threads, 0, s>>>(a);
   }
-  return check_launch("occ_decoupled_loss_fwd_bwd");
+  return check_launch("occ_decoupled_loss_fwd_bwd (stream kernel)");
 }
 
 }  // namespace occ
@@ -595,6 +1265,8 @@ extern "C" occ_status occ_decoupled_loss_fwd_bwd(
   a.adv = adv;
   a.mask = loss_mask;
   a.ws_N = (const long long*)(ws + wl.off_N);
+  a.ws_err = (int*)(ws + wl.off_err);
+  a.stage_bytes = 0;
   a.ws_loss = (float*)(ws + wl.off_loss);
   a.ws_flags = (uint8_t*)(ws + wl.off_flags);
   a.logp_out = logp_out;
@@ -612,9 +1284,9 @@ extern "C" occ_status occ_decoupled_loss_fwd_bwd(
   a.kp.denom = p->denom > 0 ? (long long)p->denom : 0;
 
   cudaStream_t s = (cudaStream_t)stream;
-  if (a.kp.denom == 0) {
+  {  // K0: N and a cleared error word (always: the workspace starts undefined)
     k0_count_valid<kK0Threads><<<1, kK0Threads, 0, s>>>(loss_mask, ids, T, V,
-                                                        (long long*)(ws + wl.off_N));
+                                                        (long long*)(ws + wl.off_N), a.ws_err);
     occ_status st = check_launch("k0_count_valid");
     if (st != OCC_OK) return st;
   }
@@ -628,7 +1300,7 @@ extern "C" occ_status occ_decoupled_loss_fwd_bwd(
       st = launch_k2<float, float>(a, vec, s);
     if (st != OCC_OK) return st;
   }
-  k2_finalize<kFinThreads><<<1, kFinThreads, 0, s>>>(T, a.ws_loss, a.ws_flags, a.ws_N, a.kp.denom,
-                                                     stats);
+  k2_finalize<kFinThreads><<<1, kFinThreads, 0, s>>>(T, a.ws_loss, a.ws_flags, a.ws_N, a.ws_err,
+                                                     a.kp.denom, stats);
   return check_launch("k2_finalize");
 }
