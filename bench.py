@@ -128,15 +128,28 @@ def kernel_source_hash():
 
 
 def ncu_traffic():
-    """Per-token / per-element DRAM bytes from the committed ncu summary, if the
-    kernels have not changed since it was captured."""
-    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    """Per-unit DRAM bytes from the committed ncu summary
+    (profiles/traffic_per_unit.json), if the kernels have not changed since it
+    was captured; {} otherwise."""
+    path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
     try:
         with open(path) as f:
             d = json.load(f)
     except Exception:
         return {}
     return d.get("kernels", {}) if d.get("source_hash") == kernel_source_hash() else {}
+
+
+def traffic_bytes(tr, name, T, n_valid, n_params):
+    """DRAM bytes of one launch, scaled from the per-unit capture."""
+    k = tr.get(name)
+    if k is None:
+        return None
+    if name == "k1_token_logprob":
+        return round(T * (k["read_per_token"] + k["write_per_token"]))
+    if name == "k2_decoupled_loss_fwd_bwd":
+        return round(n_valid * k["read_per_valid_token"] + T * k["write_per_token"])
+    return round(n_params * (k["read_per_param"] + k["write_per_param"]))
 
 
 # ----------------------------------------------------------------- the oracle arm
@@ -338,12 +351,11 @@ def main():
     }
     roof = {}
     for name, (sec, byts, units) in kern.items():
-        tr = traffic.get(name)
         achieved = byts / sec / 1e9
         roof[name] = {
             "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
             "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
-            "traffic": None if tr is None else round(tr["bytes_per_unit"] * units),
+            "traffic": traffic_bytes(traffic, name, T, n_valid, args.ewma_n),
             "algorithmic_bytes": byts, "ms": round(sec * 1e3, 4),
         }
     dominant = max(roof, key=lambda k: roof[k]["ms"])

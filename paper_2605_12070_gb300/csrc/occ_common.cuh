@@ -19,6 +19,7 @@
 namespace occ {
 
 constexpr float kLog2e = 1.4426950408889634f;  // float(log2 e)
+constexpr double kInvLog2eF = 0.6931471898132927;  // 1 / (double)kLog2e
 constexpr float kRescale = 64.f;               // lazy-rescale margin (base-2 exponent units)
 
 // ---------------------------------------------------------------- PTX helpers
@@ -239,7 +240,7 @@ __device__ __forceinline__ double lse_from(float C, float2 S) {
   const float f = frexpf(S.x, &e);  // S.x = f 2^e, f in [0.5, 1)
   const double l2 = (double)C + (double)e + (double)log2f(f) +
                     (double)(S.y / S.x) * 1.4426950408889634;
-  return l2 / (double)kLog2e;
+  return l2 * kInvLog2eF;
 }
 
 // ------------------------------------------------ mbarrier + 1-D TMA PTX

@@ -704,14 +704,17 @@ struct OutVecHint<float, 4> {
   }
 };
 
-// One CTA per row, two streaming passes (the K1 layout).  The forward pass
-// reads the row from HBM with an L2 evict-last policy; the backward pass
-// re-reads it with evict-first (its last use), so with one or two rows in
-// flight per SM the re-read is served by the 129 MB L2 and HBM sees the
-// logits once and dlogits once.  dlogits are written evict-first.
+// One CTA per row, two streaming passes (the K1 layout), with the head of the
+// row kept in shared memory.  The forward pass reads the row from HBM once:
+// its first `head` vectors are also stored in shared memory, the rest is read
+// with an L2 evict-last policy.  The backward pass takes the head from shared
+// memory and re-reads only the remainder, newest data first and with an
+// evict-first policy (its last use), so the re-read is served by L2 and HBM
+// sees the logits once and dlogits once.  dlogits are written evict-first.
 template <typename Tin, typename Tout, int NT, int U>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   constexpr int VEC = Elem<Tin>::kVec;
+  extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ RedScratch red;
   __shared__ float bc_g, bc_cb;
   const uint64_t keep = l2_policy_evict_last();
@@ -720,6 +723,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   const int64_t V = a.V;
   const int64_t nvec = V / VEC;
   const int64_t tail0 = nvec * VEC;
+  const int64_t head = min(nvec, (int64_t)(a.stage_bytes / 16));  // vectors kept on chip
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
   for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
     const int id = a.ids[row];
@@ -752,14 +756,18 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
       for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + i + u * NT, keep);
 #pragma unroll
       for (int u = 0; u < U; ++u) {
+        const int64_t ii = i + u * NT;
+        if (ii < head) head_sm[ii] = r[u];
         float x[VEC];
         Elem<Tin>::unpack(r[u], x);
         acc_add_fast(acc, x);
       }
     }
     for (; i < nvec; i += NT) {
+      const uint4 r = ld_hint_v4(zv + i, keep);
+      if (i < head) head_sm[i] = r;
       float x[VEC];
-      Elem<Tin>::unpack(ld_hint_v4(zv + i, keep), x);
+      Elem<Tin>::unpack(r, x);
       acc_add_fast(acc, x);
     }
     float xt = 0.f;
@@ -797,38 +805,32 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
         if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
       } else {
         const float sgn = g > 0.f ? -1.f : 1.f;
-        int64_t j = tid;
-        for (; j + (int64_t)(U - 1) * NT < nvec; j += (int64_t)U * NT) {
-          uint4 r[U];
-#pragma unroll
-          for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + j + u * NT, last);
-#pragma unroll
-          for (int u = 0; u < U; ++u) {
-            const int64_t jj = j + u * NT;
-            float x[VEC], d[VEC];
-            Elem<Tin>::unpack(r[u], x);
-#pragma unroll
-            for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
-            if (id >= jj * VEC && id < (jj + 1) * VEC) {
-#pragma unroll
-              for (int q = 0; q < VEC; ++q)
-                if (jj * VEC + q == id) d[q] += g;
-            }
-            OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
-          }
-        }
-        for (; j < nvec; j += NT) {
+        auto emit = [&](int64_t jj, const uint4& r) {
           float x[VEC], d[VEC];
-          Elem<Tin>::unpack(ld_hint_v4(zv + j, last), x);
+          Elem<Tin>::unpack(r, x);
 #pragma unroll
           for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
-          if (id >= j * VEC && id < (j + 1) * VEC) {
+          if (id >= jj * VEC && id < (jj + 1) * VEC) {
 #pragma unroll
             for (int q = 0; q < VEC; ++q)
-              if (j * VEC + q == id) d[q] += g;
+              if (jj * VEC + q == id) d[q] += g;
           }
-          OutVecHint<Tout, VEC>::store(drow + j * VEC, d, last);
+          OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
+        };
+        // re-read part, newest first: vectors nvec-1-tid, nvec-1-tid-NT, ... >= head
+        const int64_t nre = nvec - head;
+        int64_t k = tid;
+        for (; k + (int64_t)(U - 1) * NT < nre; k += (int64_t)U * NT) {
+          uint4 r[U];
+#pragma unroll
+          for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + (nvec - 1 - (k + u * NT)), last);
+#pragma unroll
+          for (int u = 0; u < U; ++u) emit(nvec - 1 - (k + u * NT), r[u]);
         }
+        for (; k < nre; k += NT) emit(nvec - 1 - k, ld_hint_v4(zv + (nvec - 1 - k), last));
+        // on-chip head
+#pragma unroll 4
+        for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
         if ((int64_t)tid < V - tail0) {
           float dv = sgn * ex2_approx(fmaf(xt, kLog2e, -cb));
           if (tail0 + tid == id) dv += g;
@@ -1177,14 +1179,35 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
         return launch_persistent(k2_loss_tma<Tin, Tout, 256, kK2Stages>, 256, a, pl, kK2Stages, s);
       }
     }
+    // shared-memory row head: OCC_K2_HEAD_KB overrides (0 = pure L2 re-read)
+    static const size_t head_cap = [] {
+      const char* e = getenv("OCC_K2_HEAD_KB");
+      return (size_t)(e ? atoi(e) : 80) * 1024;
+    }();
+    const size_t row_bytes = (size_t)(a.V / Elem<Tin>::kVec) * 16;
+    const size_t head_bytes = std::min(head_cap, row_bytes);
+    a.stage_bytes = (int64_t)head_bytes;
+    static const int unroll = [] {
+      const char* e = getenv("OCC_K2_UNROLL");
+      return e ? atoi(e) : 8;
+    }();
+    auto kern = (var == 3) ? k2_loss_l2<Tin, Tout, 1024, 8>
+                           : (unroll == 4 ? k2_loss_l2<Tin, Tout, 512, 4>
+                                          : (unroll == 12 ? k2_loss_l2<Tin, Tout, 512, 12>
+                                                          : k2_loss_l2<Tin, Tout, 512, 8>));
+    const int nt = (var == 3) ? 1024 : 512;
+    if (head_bytes > 0) {
+      cudaError_t e =
+          cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)head_bytes);
+      if (e != cudaSuccess)
+        return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head_bytes,
+                    cudaGetErrorString(e));
+    }
     const int64_t step = 0x7fffffffLL;
     for (int64_t r0 = 0; r0 < T; r0 += step) {
       a.row0 = r0;
       const unsigned grid = (unsigned)std::min<int64_t>(step, T - r0);
-      if (var == 3)
-        k2_loss_l2<Tin, Tout, 1024, 8><<<grid, 1024, 0, s>>>(a);
-      else
-        k2_loss_l2<Tin, Tout, 512, 8><<<grid, 512, 0, s>>>(a);
+      kern<<<grid, nt, head_bytes, s>>>(a);
     }
     return check_launch("occ_decoupled_loss_fwd_bwd");
   }
