@@ -1,10 +1,12 @@
 #!/usr/bin/env python
 """Benchmark of the decoupled off-policy correction hot path on GB300.
 
-One step = the whole path over one batch: K1 (log pi_old of the sampled tokens
-over the old logits), K0 + K2 (fused decoupled loss forward + dlogits) on the
-current logits, and K3 (PPO-EWMA update of 7.6e9 float32 proximal parameters,
-auto-reset fed by K2's statistics).  Workload: T=65536 tokens packed from 128
+One step = the whole path over one batch: log pi_old of the sampled tokens
+over the old logits, the decoupled loss forward + dlogits on the current
+logits (by default both in the one-launch occ_decoupled_loss_fused; with
+--loss-path two-call as occ_token_logprob + occ_decoupled_loss_fwd_bwd), and
+the PPO-EWMA update of 7.6e9 float32 proximal parameters, auto-reset fed by
+the loss statistics.  Workload: T=65536 tokens packed from 128
 sequences, V=151936, bf16 logits (the agentic batch), seeded synthetic data.
 Inputs (40 GB of logits, 61 GB of EWMA buffers) are far larger than L2, so no
 flush is needed between steps.
@@ -46,6 +48,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--tau", type=float, default=0.5)
     ap.add_argument("--tokens", type=int, default=None, help="resize T (profiling runs only)")
+    ap.add_argument("--loss-path", default="fused", choices=["fused", "two-call"],
+                    help="fused: one launch reads old and current logits (occ_decoupled_loss_fused); "
+                         "two-call: occ_token_logprob then occ_decoupled_loss_fwd_bwd")
     return ap.parse_args()
 
 
@@ -147,7 +152,7 @@ def traffic_bytes(tr, name, T, n_valid, n_params):
         return None
     if name == "k1_token_logprob":
         return round(T * (k["read_per_token"] + k["write_per_token"]))
-    if name == "k2_decoupled_loss_fwd_bwd":
+    if name in ("k2_decoupled_loss_fwd_bwd", "k12_decoupled_loss_fused"):
         return round(n_valid * k["read_per_valid_token"] + T * k["write_per_token"])
     return round(n_params * (k["read_per_param"] + k["write_per_param"]))
 
@@ -281,7 +286,7 @@ def main():
     denom = dp.global_token_count(n_valid) if world > 1 else 0
     stream = torch.cuda.current_stream(dev)
 
-    def step(ev=None):
+    def loss_two_call(ev=None):
         if ev is not None:
             ev[0].record(stream)
         occ.occ_token_logprob(batch.z_old, batch.ids, logp_out=lp_old)
@@ -291,6 +296,20 @@ def main():
                                        batch.mask, **batch.thresholds(), denom=denom,
                                        dlogits=dlogits, logp_out=logp, flags_out=flags,
                                        stats=stats, workspace=ws)
+
+    def loss_fused(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+            ev[1].record(stream)
+        occ.occ_decoupled_loss_fused(batch.z_theta, batch.z_old, batch.ids, batch.logp_mu,
+                                     batch.adv, batch.mask, **batch.thresholds(), denom=denom,
+                                     dlogits=dlogits, logp_out=logp, logp_old_out=lp_old,
+                                     flags_out=flags, stats=stats, workspace=ws)
+
+    loss = loss_fused if args.loss_path == "fused" else loss_two_call
+
+    def step(ev=None, loss_fn=None):
+        (loss_fn or loss)(ev)
         if world > 1:
             dp.allreduce_loss_stats(stats)
         if ev is not None:
@@ -335,20 +354,42 @@ def main():
     k2 = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps / 1e3
     k3 = sum(e[2].elapsed_time(e[3]) for e in evs) / args.steps / 1e3
     ms_step = elapsed / args.steps * 1e3
+    resets = occ.decode_ewma_state(state).n_resets - resets_before
+
+    # the other loss path, timed the same way on the same inputs (breakdown only)
+    alt_fn = loss_two_call if args.loss_path == "fused" else loss_fused
+    for _ in range(2):
+        step(loss_fn=alt_fn)
+    aevs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(10)]
+    for k in range(10):
+        step(aevs[k], loss_fn=alt_fn)
+    torch.cuda.synchronize()
+    alt_k1 = sum(e[0].elapsed_time(e[1]) for e in aevs) / 10 / 1e3
+    alt_k2 = sum(e[1].elapsed_time(e[2]) for e in aevs) / 10 / 1e3
 
     peak, peak_kind = measured_peak()
     traffic = ncu_traffic()
     bytes_k1 = T * V * 2 + T * 8
     bytes_k2 = n_valid * V * 2 + T * V * 2 + T * 37
-    resets = occ.decode_ewma_state(state).n_resets - resets_before
+    bytes_fused = 2 * n_valid * V * 2 + T * V * 2 + T * 41
     # a regular update reads theta_prox and theta and writes theta_prox; a reset copies theta
     bytes_k3 = args.ewma_n * (12 * (args.steps - resets) + 8 * resets) // args.steps
     st_last = occ.decode_loss_stats(stats)
-    kern = {
-        "k1_token_logprob": (k1, bytes_k1, T),
-        "k2_decoupled_loss_fwd_bwd": (k2, bytes_k2, T),
-        "k3_ewma_update": (k3, bytes_k3, args.ewma_n),
-    }
+    if args.loss_path == "fused":
+        kern = {"k12_decoupled_loss_fused": (k2, bytes_fused, T),
+                "k3_ewma_update": (k3, bytes_k3, args.ewma_n)}
+        alt = {"path": "two-call", "ms": round((alt_k1 + alt_k2) * 1e3, 4),
+               "k1_ms": round(alt_k1 * 1e3, 4), "k2_ms": round(alt_k2 * 1e3, 4),
+               "tokens_per_s": round(world * T / (alt_k1 + alt_k2), 1),
+               "hbm_frac": round((bytes_k1 + bytes_k2) / (alt_k1 + alt_k2) / 1e9 / peak, 4)}
+        loss_bytes = bytes_fused
+    else:
+        kern = {"k1_token_logprob": (k1, bytes_k1, T), "k2_decoupled_loss_fwd_bwd": (k2, bytes_k2, T),
+                "k3_ewma_update": (k3, bytes_k3, args.ewma_n)}
+        alt = {"path": "fused", "ms": round(alt_k2 * 1e3, 4),
+               "tokens_per_s": round(world * T / alt_k2, 1),
+               "hbm_frac": round(bytes_fused / alt_k2 / 1e9 / peak, 4)}
+        loss_bytes = bytes_k1 + bytes_k2
     roof = {}
     for name, (sec, byts, units) in kern.items():
         achieved = byts / sec / 1e9
@@ -375,9 +416,10 @@ def main():
         "data": "synthetic",
         "config": {
             "workload": (f"decoupled-loss step on T={T} tokens (128 packed sequences, "
-                         f"{n_valid} valid), V={V} bf16 logits (K1 old log-probs + K0/K2 fused "
-                         f"loss fwd+bwd) chained with the PPO-EWMA update of "
-                         f"{args.ewma_n} fp32 parameters (K3)"),
+                         f"{n_valid} valid), V={V} bf16 old and current logits (log pi_old, "
+                         f"loss fwd + dlogits) chained with the PPO-EWMA update of "
+                         f"{args.ewma_n} fp32 parameters"),
+            "loss_path": args.loss_path,
             "T": T, "V": V, "ewma_params": args.ewma_n, "logits_dtype": "bf16",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": "inputs larger than L2 (40 GB logits, 61 GB EWMA buffers): no flush",
@@ -386,16 +428,17 @@ def main():
         },
         "roofline": dict(roof[dominant], kernel=dominant),
         "kernels": roof,
-        "loss_only": {"tokens_per_s": round(world * T / ((k1 + k2)), 1), "ms": round(loss_ms, 4),
-                      "hbm_frac": round((bytes_k1 + bytes_k2) / (k1 + k2) / 1e9 / peak, 4)},
-        "gpu_launches": args.steps * 6,
+        "loss_only": {"path": args.loss_path, "tokens_per_s": round(world * T / (k1 + k2), 1),
+                      "ms": round(loss_ms, 4),
+                      "hbm_frac": round(loss_bytes / (k1 + k2) / 1e9 / peak, 4)},
+        "loss_only_other_path": alt,
+        "gpu_launches": args.steps * (5 if args.loss_path == "fused" else 6),
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(batch, args.ewma_n, args.cpu_seconds)
     if not args.no_e2e:
-        line["e2e"] = run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits,
-                              logp, flags, denom, world, dev)
+        line["e2e"] = run_e2e(args, batch, theta, theta_prox, state, stats, loss, world, dev)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -413,8 +456,7 @@ def _host_available_bytes():
     return 0
 
 
-def run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits, logp, flags, denom,
-            world, dev):
+def run_e2e(args, batch, theta, theta_prox, state, stats, loss_fn, world, dev):
     """Same step through the public API with the inputs in pinned HOST memory:
     every step copies the logits, token arrays and the new actor parameters to
     the device and reads the loss statistics back."""
@@ -437,11 +479,7 @@ def run_e2e(args, batch, theta, theta_prox, state, stats, ws, lp_old, dlogits, l
     def e2e_step():
         for h, d in zip(host, dev_inputs):
             d.copy_(h, non_blocking=True)
-        occ.occ_token_logprob(batch.z_old, batch.ids, logp_out=lp_old)
-        occ.occ_decoupled_loss_fwd_bwd(batch.z_theta, batch.ids, lp_old, batch.logp_mu, batch.adv,
-                                       batch.mask, **batch.thresholds(), denom=denom,
-                                       dlogits=dlogits, logp_out=logp, flags_out=flags,
-                                       stats=stats, workspace=ws)
+        loss_fn()
         if world > 1:
             dp.allreduce_loss_stats(stats)
         occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=args.tau)

@@ -161,6 +161,37 @@ occ_status occ_decoupled_loss_fwd_bwd(const void* logits, occ_dtype dt, int64_t 
                                       size_t ws_bytes, void* stream);
 
 /*
+ * occ_decoupled_loss_fused -- occ_token_logprob on the old logits and
+ * occ_decoupled_loss_fwd_bwd on the current logits in one launch.
+ *
+ * Each token's old row (pi_old, or the proxy pi_prox of Eq. 5 / pi_async of
+ * Table 1) and current row are streamed by the same CTA, so log pi_old(y_t)
+ * never leaves the kernel and enters the r_d / r_s decisions (Eqs. 1-4) in
+ * float64; the old row of a dropped token (mask 0 or bad id) is not read.
+ * Results equal the two-call sequence up to that float32 rounding of log pi_old.
+ * Optionally, in the same pass and with no extra memory traffic, per-token
+ * diagnostics of the proximal reference's lag (Sec. 5.2, App. D):
+ *   entropy_out[t] = H(pi_theta(.|t)) = lse - sum_v p_v z_v
+ *   kl_out[t]      = KL(pi_old(.|t) || pi_theta(.|t))
+ * (both 0 for dropped tokens).
+ *
+ *   logits_old   [T, ld_old], same dtype as logits, ld_old >= V
+ *   logp_old_out [T] float32 or NULL: log pi_old(y_t) of valid tokens (0 for dropped,
+ *                NaN for a bad id)
+ *   entropy_out, kl_out [T] float32 or NULL
+ * Every other argument is as in occ_decoupled_loss_fwd_bwd (the same workspace size);
+ * dlogits must not overlap logits_old.
+ */
+occ_status occ_decoupled_loss_fused(const void* logits, const void* logits_old, occ_dtype dt,
+                                    int64_t T, int64_t V, int64_t ld, int64_t ld_old,
+                                    const int32_t* ids, const float* logp_mu, const float* adv,
+                                    const uint8_t* loss_mask, const occ_loss_params* p,
+                                    float* logp_out, float* logp_old_out, uint8_t* flags_out,
+                                    float* entropy_out, float* kl_out, void* dlogits,
+                                    int64_t ld_grad, occ_loss_stats* stats, void* workspace,
+                                    size_t ws_bytes, void* stream);
+
+/*
  * occ_decoupled_loss_fwd_bwd_noalloc -- occ_decoupled_loss_fwd_bwd without a
  * caller-supplied workspace.  (The paper has no counterpart: this is an
  * interface convenience.)

@@ -1,0 +1,449 @@
+// K1 + K2 fused: log pi_old, the decoupled loss and dlogits in one launch,
+// with optional per-token diagnostics of the proximal reference.
+//
+// One CTA per row streams the old (or proxy) logits row and the current
+// logits row side by side in the forward pass: log pi_old(y_t) and
+// log pi_theta(y_t) come out of the same CTA (Eq. 1 factors), log pi_old stays
+// in float64 into the ratio decisions (Eqs. 2-4), and the old row of a dropped
+// token is never read.  The backward pass is the K2 one (the current row's
+// head from shared memory, the rest re-read from L2).
+//
+// Diagnostics (optional, no extra HBM bytes): the entropy of pi_theta,
+// H = lse - E_p[z], and KL(pi_old || pi_theta) = E_{p_old}[z_old - z] -
+// lse_old + lse, which track the reference-policy lag that the revised
+// PPO-EWMA is built to limit (Sec. 5.2, App. D).
+#include "occ_loss_common.cuh"
+
+namespace occ {
+
+// Online (c, s, sv): s = sum 2^(x L - c), sv = sum 2^(x L - c) v.
+struct LseAccV {
+  float c, s, sv;
+};
+
+template <int N, bool WV>
+__device__ __forceinline__ void accv_add(LseAccV& a, const float (&x)[N], const float (&v)[N]) {
+  float t = 0.f, tv = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    const float e = ex2_approx(fmaf(x[j], kLog2e, -a.c));
+    t += e;
+    if (WV) tv = fmaf(e, v[j], tv);
+  }
+  if (t <= 1.8446744073709552e19f) {  // 2^64; false for inf / NaN and for c = -inf
+    a.s += t;
+    a.sv += tv;
+    return;
+  }
+  float m = x[0];
+#pragma unroll
+  for (int j = 1; j < N; ++j) m = fmaxf(m, x[j]);
+  const float ms = m * kLog2e;
+  if (ms > a.c + kRescale) {
+    const float f = exp2f(a.c - ms);
+    a.s *= f;
+    a.sv *= f;
+    a.c = ms;
+  }
+  if (a.c == -INFINITY) return;
+  t = 0.f;
+  tv = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    const float e = ex2_approx(fmaf(x[j], kLog2e, -a.c));
+    t += e;
+    if (WV) tv = fmaf(e, v[j], tv);
+  }
+  a.s += t;
+  a.sv += tv;
+}
+
+struct FusedRed {
+  float c[2][32];
+  float2 s[2][32];
+  float sv[2][32];
+};
+
+// Block merge of two accumulators; the results are valid in thread 0.
+template <int NT>
+__device__ __forceinline__ void block_lse_v2(const LseAccV (&acc)[2], FusedRed& r, float (&C)[2],
+                                             float2 (&S)[2], float (&SV)[2]) {
+  constexpr int NW = NT / 32;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const float wm = warp_max(acc[k].c);
+    const float f = acc[k].c == -INFINITY ? 0.f : exp2f(acc[k].c - wm);
+    float2 v = warp_pair_sum(make_float2(acc[k].s * f, 0.f));
+    float sv = acc[k].sv * f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, o);
+    if (lane == 0) {
+      r.c[k][wid] = wm;
+      r.s[k][wid] = v;
+      r.sv[k][wid] = sv;
+    }
+  }
+  __syncthreads();
+  if (wid == 0) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const float cw = lane < NW ? r.c[k][lane] : -INFINITY;
+      const float cm = warp_max(cw);
+      float2 w = make_float2(0.f, 0.f);
+      float sv = 0.f;
+      if (lane < NW && cw != -INFINITY) {
+        const float f = exp2f(cw - cm);
+        const float2 p = r.s[k][lane];
+        const float hi = p.x * f;
+        w = make_float2(hi, fmaf(p.x, f, -hi) + p.y * f);
+        sv = r.sv[k][lane] * f;
+      }
+      w = warp_pair_sum(w);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, o);
+      C[k] = cm;
+      S[k] = w;
+      SV[k] = sv;
+    }
+  }
+}
+
+struct FusedArgs {
+  K2Args a;
+  const void* logits_old;
+  int64_t ld_old;
+  float* logp_old_out;
+  float* entropy_out;
+  float* kl_out;
+};
+
+__device__ __forceinline__ void fused_dropped_outputs(const FusedArgs& f, int64_t row, bool m,
+                                                      bool id_ok) {
+  dropped_token_outputs(f.a, row, m, id_ok);
+  if (f.logp_old_out) f.logp_old_out[row] = id_ok ? 0.f : __int_as_float(0x7fc00000);
+  if (f.entropy_out) f.entropy_out[row] = 0.f;
+  if (f.kl_out) f.kl_out[row] = 0.f;
+}
+
+// Thread 0: token scalars from the two merged rows.  Writes the per-token
+// outputs and returns (g, cb) for the backward pass.
+__device__ __forceinline__ void fused_token_epilogue(const FusedArgs& f, int64_t row,
+                                                     const float (&C)[2], const float2 (&S)[2],
+                                                     const float (&SV)[2], float zy, float zyo,
+                                                     float lpm, float A, long long N, float& g,
+                                                     float& cb) {
+  const K2Args& a = f.a;
+  const double lse = lse_from(C[0], S[0]);
+  const double lse_old = lse_from(C[1], S[1]);
+  const double logp_old = (double)zyo - lse_old;
+  float loss_t, logp_f;
+  uint32_t fl;
+  token_math(a.kp, lse, zy, logp_old, lpm, A, N, g, loss_t, fl, logp_f);
+  cb = 0.f;
+  if (g != 0.f) {
+    int e;
+    const float fm = frexpf(fabsf(g), &e);
+    cb = (float)(lse * (double)kLog2e - (double)e - (double)log2f(fm));
+  }
+  a.ws_loss[row] = loss_t;
+  a.ws_flags[row] = (uint8_t)fl;
+  if (a.logp_out) a.logp_out[row] = logp_f;
+  if (a.flags_out) a.flags_out[row] = (uint8_t)fl;
+  if (f.logp_old_out) f.logp_old_out[row] = (float)logp_old;
+  if (f.entropy_out) {
+    const double ez = (double)SV[0] / ((double)S[0].x + (double)S[0].y);
+    f.entropy_out[row] = (float)(lse - ez);
+  }
+  if (f.kl_out) {
+    const double ed = (double)SV[1] / ((double)S[1].x + (double)S[1].y);
+    f.kl_out[row] = (float)(ed - lse_old + lse);
+  }
+}
+
+// Vector path: 16-byte rows.  U vectors of each row in flight per thread.
+template <typename Tin, typename Tout, int NT, int U, bool DIAG>
+__global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
+  constexpr int VEC = Elem<Tin>::kVec;
+  extern __shared__ __align__(16) uint4 head_sm[];
+  __shared__ FusedRed red;
+  __shared__ float bc_g, bc_cb;
+  const K2Args& a = f.a;
+  const uint64_t keep = l2_policy_evict_last();
+  const uint64_t last = l2_policy_evict_first();
+  const int tid = threadIdx.x;
+  const int64_t V = a.V;
+  const int64_t nvec = V / VEC;
+  const int64_t tail0 = nvec * VEC;
+  const int64_t head = min(nvec, (int64_t)(a.stage_bytes / 16));
+  const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
+  for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
+    const int id = a.ids[row];
+    const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
+    const bool id_ok = id >= 0 && (int64_t)id < V;
+    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    if (!(m && id_ok)) {
+      if (drow) {
+        for (int64_t i = tid; i < nvec; i += NT) OutVecHint<Tout, VEC>::zero(drow + i * VEC, last);
+        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+      }
+      if (tid == 0) fused_dropped_outputs(f, row, m, id_ok);
+      continue;
+    }
+    const Tin* z = (const Tin*)a.logits + row * a.ld;
+    const Tin* zo = (const Tin*)f.logits_old + row * f.ld_old;
+    float zy = 0.f, zyo = 0.f, lpm = 0.f, A = 0.f;
+    if (tid == 0) {
+      zy = Elem<Tin>::load(z + id);
+      zyo = Elem<Tin>::load(zo + id);
+      lpm = a.lp_mu[row];
+      A = a.adv[row];
+    }
+    const uint4* zv = reinterpret_cast<const uint4*>(z);
+    const uint4* zov = reinterpret_cast<const uint4*>(zo);
+    LseAccV acc[2] = {{-INFINITY, 0.f, 0.f}, {-INFINITY, 0.f, 0.f}};
+    auto consume = [&](int64_t ii, const uint4& rt, const uint4& ro) {
+      if (ii < head) head_sm[ii] = rt;
+      float x[VEC], xo[VEC], d[VEC];
+      Elem<Tin>::unpack(rt, x);
+      Elem<Tin>::unpack(ro, xo);
+      if (DIAG) {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) d[q] = xo[q] - x[q];
+      }
+      accv_add<VEC, DIAG>(acc[0], x, x);
+      accv_add<VEC, DIAG>(acc[1], xo, d);
+    };
+    int64_t i = tid;
+    for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
+      uint4 rt[U], ro[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        rt[u] = ld_hint_v4(zv + i + u * NT, keep);
+        ro[u] = ld_hint_v4(zov + i + u * NT, last);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) consume(i + u * NT, rt[u], ro[u]);
+    }
+    for (; i < nvec; i += NT) consume(i, ld_hint_v4(zv + i, keep), ld_hint_v4(zov + i, last));
+    float xt = 0.f;
+    if ((int64_t)tid < V - tail0) {
+      xt = Elem<Tin>::load(z + tail0 + tid);
+      const float xot = Elem<Tin>::load(zo + tail0 + tid);
+      float x1[1] = {xt}, xo1[1] = {xot}, d1[1] = {xot - xt};
+      accv_add<1, DIAG>(acc[0], x1, x1);
+      accv_add<1, DIAG>(acc[1], xo1, d1);
+    }
+    float C[2], SV[2];
+    float2 S[2];
+    block_lse_v2<NT>(acc, red, C, S, SV);
+    if (tid == 0) {
+      float g, cb;
+      fused_token_epilogue(f, row, C, S, SV, zy, zyo, lpm, A, N, g, cb);
+      bc_g = g;
+      bc_cb = cb;
+    }
+    __syncthreads();
+    if (drow) {
+      const float g = bc_g, cb = bc_cb;
+      if (g == 0.f) {
+        for (int64_t j = tid; j < nvec; j += NT) OutVecHint<Tout, VEC>::zero(drow + j * VEC, last);
+        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+      } else {
+        const float sgn = g > 0.f ? -1.f : 1.f;
+        auto emit = [&](int64_t jj, const uint4& r) {
+          float x[VEC], d[VEC];
+          Elem<Tin>::unpack(r, x);
+#pragma unroll
+          for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
+          if (id >= jj * VEC && id < (jj + 1) * VEC) {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q)
+              if (jj * VEC + q == id) d[q] += g;
+          }
+          OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
+        };
+        const int64_t nre = nvec - head;
+        int64_t k = tid;
+        for (; k + (int64_t)(2 * U - 1) * NT < nre; k += (int64_t)2 * U * NT) {
+          uint4 r[2 * U];
+#pragma unroll
+          for (int u = 0; u < 2 * U; ++u) r[u] = ld_hint_v4(zv + (nvec - 1 - (k + u * NT)), last);
+#pragma unroll
+          for (int u = 0; u < 2 * U; ++u) emit(nvec - 1 - (k + u * NT), r[u]);
+        }
+        for (; k < nre; k += NT) emit(nvec - 1 - k, ld_hint_v4(zv + (nvec - 1 - k), last));
+#pragma unroll 4
+        for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
+        if ((int64_t)tid < V - tail0) {
+          float dv = sgn * ex2_approx(fmaf(xt, kLog2e, -cb));
+          if (tail0 + tid == id) dv += g;
+          out_scalar(drow + tail0 + tid, dv);
+        }
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Any alignment: element loads, old and current rows in one pass, then the
+// backward pass over global memory.
+template <typename Tin, typename Tout, int NT, bool DIAG>
+__global__ void __launch_bounds__(NT) k2_fused_stream(const FusedArgs f) {
+  __shared__ FusedRed red;
+  __shared__ float bc_g, bc_cb;
+  const K2Args& a = f.a;
+  const int tid = threadIdx.x;
+  const int64_t V = a.V;
+  const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
+  for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
+    const int id = a.ids[row];
+    const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
+    const bool id_ok = id >= 0 && (int64_t)id < V;
+    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    if (!(m && id_ok)) {
+      if (drow)
+        for (int64_t v = tid; v < V; v += NT) out_scalar(drow + v, 0.f);
+      if (tid == 0) fused_dropped_outputs(f, row, m, id_ok);
+      continue;
+    }
+    const Tin* z = (const Tin*)a.logits + row * a.ld;
+    const Tin* zo = (const Tin*)f.logits_old + row * f.ld_old;
+    float zy = 0.f, zyo = 0.f, lpm = 0.f, A = 0.f;
+    if (tid == 0) {
+      zy = Elem<Tin>::load(z + id);
+      zyo = Elem<Tin>::load(zo + id);
+      lpm = a.lp_mu[row];
+      A = a.adv[row];
+    }
+    LseAccV acc[2] = {{-INFINITY, 0.f, 0.f}, {-INFINITY, 0.f, 0.f}};
+    for (int64_t v0 = tid; v0 < V; v0 += 8 * (int64_t)NT) {
+      float x[8], xo[8], xv[8], d[8];  // padding: weight 0 and value 0
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int64_t v = v0 + (int64_t)j * NT;
+        x[j] = v < V ? Elem<Tin>::load(z + v) : -INFINITY;
+        xo[j] = v < V ? Elem<Tin>::load(zo + v) : -INFINITY;
+        xv[j] = v < V ? x[j] : 0.f;
+        d[j] = v < V ? xo[j] - x[j] : 0.f;
+      }
+      accv_add<8, DIAG>(acc[0], x, xv);
+      accv_add<8, DIAG>(acc[1], xo, d);
+    }
+    float C[2], SV[2];
+    float2 S[2];
+    block_lse_v2<NT>(acc, red, C, S, SV);
+    if (tid == 0) {
+      float g, cb;
+      fused_token_epilogue(f, row, C, S, SV, zy, zyo, lpm, A, N, g, cb);
+      bc_g = g;
+      bc_cb = cb;
+    }
+    __syncthreads();
+    if (drow) {
+      const float g = bc_g, cb = bc_cb;
+      const float sgn = g > 0.f ? -1.f : 1.f;
+      for (int64_t v = tid; v < V; v += NT) {
+        float dv = 0.f;
+        if (g != 0.f) {
+          dv = sgn * ex2_approx(fmaf(Elem<Tin>::load(z + v), kLog2e, -cb));
+          if (v == id) dv += g;
+        }
+        out_scalar(drow + v, dv);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+constexpr int kFusedThreads = 512;
+constexpr int kFusedUnroll = 4;
+constexpr size_t kFusedHeadBytes = 80 * 1024;
+
+template <typename Tin, typename Tout, bool DIAG>
+static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
+  const int64_t T = f.a.T;
+  const int64_t step = 0x7fffffffLL;
+  if (vec) {
+    const size_t row_bytes = (size_t)(f.a.V / Elem<Tin>::kVec) * 16;
+    const size_t head = std::min(kFusedHeadBytes, row_bytes);
+    f.a.stage_bytes = (int64_t)head;
+    auto kern = k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, DIAG>;
+    if (head > 0) {
+      cudaError_t e =
+          cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)head);
+      if (e != cudaSuccess)
+        return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head,
+                    cudaGetErrorString(e));
+    }
+    for (int64_t r0 = 0; r0 < T; r0 += step) {
+      f.a.row0 = r0;
+      kern<<<(unsigned)std::min<int64_t>(step, T - r0), kFusedThreads, head, s>>>(f);
+    }
+  } else {
+    for (int64_t r0 = 0; r0 < T; r0 += step) {
+      f.a.row0 = r0;
+      k2_fused_stream<Tin, Tout, kFusedThreads, DIAG>
+          <<<(unsigned)std::min<int64_t>(step, T - r0), kFusedThreads, 0, s>>>(f);
+    }
+  }
+  return check_launch("occ_decoupled_loss_fused");
+}
+
+template <typename Tin, typename Tout>
+static occ_status launch_fused_any(const FusedArgs& f, bool vec, bool diag, cudaStream_t s) {
+  return diag ? launch_fused<Tin, Tout, true>(f, vec, s) : launch_fused<Tin, Tout, false>(f, vec, s);
+}
+
+}  // namespace occ
+
+using namespace occ;
+
+extern "C" occ_status occ_decoupled_loss_fused(
+    const void* logits, const void* logits_old, occ_dtype dt, int64_t T, int64_t V, int64_t ld,
+    int64_t ld_old, const int32_t* ids, const float* logp_mu, const float* adv,
+    const uint8_t* loss_mask, const occ_loss_params* p, float* logp_out, float* logp_old_out,
+    uint8_t* flags_out, float* entropy_out, float* kl_out, void* dlogits, int64_t ld_grad,
+    occ_loss_stats* stats, void* workspace, size_t ws_bytes, void* stream) {
+  clear_error();
+  FusedArgs f;
+  bool vec = false;
+  occ_status st = prepare_loss_args(logits, dt, T, V, ld, ids, logp_mu, adv, loss_mask, p,
+                                    logp_out, flags_out, dlogits, ld_grad, stats, workspace,
+                                    ws_bytes, f.a, vec);
+  if (st != OCC_OK) return st;
+  const size_t es = dtype_size(dt);
+  if (T > 0) {
+    if (!logits_old) return fail(OCC_ERR_INVALID_ARG, "null logits_old");
+    if (ld_old < V) return fail(OCC_ERR_INVALID_ARG, "ld_old < V");
+    if (!aligned(logits_old, es) || (logp_old_out && !aligned(logp_old_out, 4)) ||
+        (entropy_out && !aligned(entropy_out, 4)) || (kl_out && !aligned(kl_out, 4)))
+      return fail(OCC_ERR_MISALIGNED, "arrays must be aligned to their element size");
+    if (dlogits) {
+      const size_t es_out = p->dlogits_f32 ? 4 : es;
+      const size_t old_bytes = ((size_t)(T - 1) * (size_t)ld_old + (size_t)V) * es;
+      const size_t out_bytes = ((size_t)(T - 1) * (size_t)ld_grad + (size_t)V) * es_out;
+      if (overlaps(logits_old, old_bytes, dlogits, out_bytes))
+        return fail(OCC_ERR_INVALID_ARG, "dlogits overlaps logits_old");
+    }
+    vec = vec && aligned(logits_old, 16) && ((ld_old * (int64_t)es) % 16 == 0);
+  }
+  f.logits_old = logits_old;
+  f.ld_old = ld_old;
+  f.logp_old_out = logp_old_out;
+  f.entropy_out = entropy_out;
+  f.kl_out = kl_out;
+  cudaStream_t s = (cudaStream_t)stream;
+  st = launch_k0(f.a, s);
+  if (st != OCC_OK) return st;
+  if (T > 0) {
+    const bool diag = entropy_out || kl_out;
+    if (dt == OCC_BF16)
+      st = p->dlogits_f32 ? launch_fused_any<bf16_t, float>(f, vec, diag, s)
+                          : launch_fused_any<bf16_t, bf16_t>(f, vec, diag, s);
+    else
+      st = launch_fused_any<float, float>(f, vec, diag, s);
+    if (st != OCC_OK) return st;
+  }
+  return launch_finalize(f.a, stats, s);
+}

@@ -32,7 +32,7 @@ _STATE_FMT = "<3d4i"
 
 # Every symbol declared in include/occ.h.
 EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_fwd_bwd",
-           "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update", "occ_ewma_state_init",
+           "occ_decoupled_loss_fused", "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update", "occ_ewma_state_init",
            "occ_status_string", "occ_last_error", "occ_version")
 
 
@@ -69,6 +69,10 @@ def lib():
                                              ctypes.POINTER(LossParams), vp, vp, vp, i64, vp, vp,
                                              ctypes.c_size_t, vp]
     L.occ_decoupled_loss_fwd_bwd.restype = i32
+    L.occ_decoupled_loss_fused.argtypes = [vp, vp, i32, i64, i64, i64, i64, vp, vp, vp, vp,
+                                           ctypes.POINTER(LossParams), vp, vp, vp, vp, vp, vp, i64,
+                                           vp, vp, ctypes.c_size_t, vp]
+    L.occ_decoupled_loss_fused.restype = i32
     L.occ_decoupled_loss_fwd_bwd_noalloc.argtypes = [vp, i32, i64, i64, i64, vp, vp, vp, vp, vp,
                                                      ctypes.POINTER(LossParams), vp, vp, vp, i64,
                                                      vp, vp]
@@ -215,6 +219,59 @@ def occ_decoupled_loss_fwd_bwd(logits, ids, logp_old, logp_mu, adv, loss_mask=No
         _stream(stream, dev))
     _check(rc, "occ_decoupled_loss_fwd_bwd")
     return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "flags": flags_out}
+
+
+def occ_decoupled_loss_fused(logits, logits_old, ids, logp_mu, adv, loss_mask=None, *, rd_lo,
+                             rd_hi, eps_low, eps_high, rd_weight=1, grad_scale=1.0, denom=0,
+                             dlogits_f32=False, dlogits="new", logp_out=None, logp_old_out=None,
+                             flags_out=None, entropy_out=None, kl_out=None, want_logp=True,
+                             want_logp_old=True, want_flags=True, want_diagnostics=False,
+                             stats=None, workspace=None, stream=None):
+    """log pi_old and the decoupled loss (+ dlogits) in one launch; optional
+    per-token entropy of pi_theta and KL(pi_old || pi_theta)."""
+    _cuda(logits, logits_old, ids, logp_mu, adv, loss_mask)
+    T, V, ld = _rows(logits)
+    To, Vo, ld_old = _rows(logits_old)
+    if (To, Vo) != (T, V) or logits_old.dtype != logits.dtype:
+        raise OccError("logits_old must match logits in shape and dtype")
+    dev = logits.device
+    out_dtype = torch.float32 if (dlogits_f32 or logits.dtype == torch.float32) else logits.dtype
+    if isinstance(dlogits, str):
+        if dlogits == "new":
+            dlogits = torch.empty((T, V), dtype=out_dtype, device=dev)
+        elif dlogits == "inplace":
+            dlogits = logits
+        else:
+            raise OccError(f"dlogits={dlogits!r}")
+    if dlogits is not None:
+        _cuda(dlogits)
+        if dlogits.dim() != 2 or dlogits.stride(1) != 1 or dlogits.dtype != out_dtype:
+            raise OccError("dlogits must be 2-D, unit column stride, dtype " + str(out_dtype))
+    ld_grad = dlogits.stride(0) if dlogits is not None else 0
+
+    def _f32(t, want):
+        return torch.empty(T, dtype=torch.float32, device=dev) if (t is None and want) else t
+
+    logp_out = _f32(logp_out, want_logp)
+    logp_old_out = _f32(logp_old_out, want_logp_old)
+    entropy_out = _f32(entropy_out, want_diagnostics)
+    kl_out = _f32(kl_out, want_diagnostics)
+    if flags_out is None and want_flags:
+        flags_out = torch.empty(T, dtype=torch.uint8, device=dev)
+    if stats is None:
+        stats = new_loss_stats(dev)
+    if workspace is None:
+        workspace = new_workspace(T, V, dev)
+    p = LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
+                   float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)))
+    rc = lib().occ_decoupled_loss_fused(
+        _ptr(logits), _ptr(logits_old), _dtype_code(logits), T, V, ld, ld_old, _ptr(ids),
+        _ptr(logp_mu), _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out),
+        _ptr(logp_old_out), _ptr(flags_out), _ptr(entropy_out), _ptr(kl_out), _ptr(dlogits),
+        ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(), _stream(stream, dev))
+    _check(rc, "occ_decoupled_loss_fused")
+    return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "logp_old": logp_old_out,
+            "flags": flags_out, "entropy": entropy_out, "kl": kl_out}
 
 
 NOALLOC_MAX_TOKENS = 786432  # OCC_NOALLOC_MAX_TOKENS
