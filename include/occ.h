@@ -73,7 +73,21 @@ typedef struct {
   int32_t rd_weight;        /* 1: token weight M(r_d) r_d (Table 5, "PPO-EWMA & train_infer");
                                0: weight M(r_d) only (Table 5, "decoupled PPO & train_infer")  */
   int32_t dlogits_f32;      /* 1: write float32 dlogits even for bf16 logits                   */
+  int32_t proxy;            /* source of log pi_old (Table 1 proxies, App. A):
+                               OCC_PROXY_NONE: the logp_old argument (pi_old, pi_prox of Eq. 5 or
+                                 pi_async computed from their own logits);
+                               OCC_PROXY_LOGLINEAR: log pi_prox = alpha log mu_old +
+                                 (1 - alpha) log pi_theta, per token;
+                               OCC_PROXY_ARITHMETIC: pi_prox = alpha mu_old + (1 - alpha) pi_theta
+                                 ("linear_prox"), per token.
+                               A proxy is a constant in the gradient (not differentiated). */
+  int32_t reserved;
+  double alpha;             /* behaviour-policy weight of the proxy, in [0, 1]              */
 } occ_loss_params;
+
+#define OCC_PROXY_NONE 0
+#define OCC_PROXY_LOGLINEAR 1
+#define OCC_PROXY_ARITHMETIC 2
 
 /* Loss results (DEVICE struct, fully written by every successful call). */
 typedef struct {
@@ -138,7 +152,8 @@ size_t occ_loss_workspace_bytes(int64_t T, int64_t V);
  * Threshold decisions are taken in log-ratio space in float64.
  *
  *   logits     [T, ld] bf16 or f32 (dt); read once
- *   ids        [T] int32;  logp_old, logp_mu, adv: [T] float32
+ *   ids        [T] int32;  logp_old, logp_mu, adv: [T] float32 (logp_old may be NULL when
+ *              p->proxy != OCC_PROXY_NONE: log pi_old is then built from logp_mu and logp_t)
  *   loss_mask  [T] uint8 or NULL (= all ones)
  *   p          HOST pointer to the options
  *   logp_out   [T] float32 or NULL: logp_t for valid tokens, 0 for dropped ones

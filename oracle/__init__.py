@@ -21,6 +21,8 @@ loss   -- R1..R9: logsumexp/log-prob (Eq. 1 factors), the r_d band mask (Eq. 4),
           the sign-dependent PPO clip (Eqs. 2-3), token-mean loss, gradient.
 ewma   -- R10: the revised PPO-EWMA proximal parameters (Eq. 5, App. B),
           the staleness-aware decay rule and the auto-reset rule (Sec. 5.2).
+proxies -- R12: the log-linear and arithmetic interpolation proxies of
+          Table 1 / App. A that stand in for a missing pi_old.
 diagnostics -- R11: per-token entropy of pi_theta and KL(pi_old || pi_theta),
           the reference-lag diagnostics (Sec. 5.2, App. D).
 rows   -- chunking / threading driver (no arithmetic of the method).
@@ -34,5 +36,6 @@ from .loss import LossParams, token_logprob, token_terms, decoupled_loss, softma
     FLAG_IN_BAND, \
     FLAG_CLIPPED, FLAG_ACTIVE, FLAG_VALID  # noqa: F401
 from .diagnostics import token_entropy, token_kl  # noqa: F401
+from .proxies import proxy_logprob  # noqa: F401
 from .ewma import EwmaState, ewma_coefficients, ewma_update, ewma_closed_form, \
     beta_for_window, center_of_mass  # noqa: F401

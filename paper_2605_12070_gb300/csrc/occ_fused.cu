@@ -412,6 +412,10 @@ extern "C" occ_status occ_decoupled_loss_fused(
                                     logp_out, flags_out, dlogits, ld_grad, stats, workspace,
                                     ws_bytes, f.a, vec);
   if (st != OCC_OK) return st;
+  if (p->proxy != OCC_PROXY_NONE)
+    return fail(OCC_ERR_INVALID_ARG,
+                "the fused kernel takes log pi_old from logits_old; proxies are a mode of "
+                "occ_decoupled_loss_fwd_bwd");
   const size_t es = dtype_size(dt);
   if (T > 0) {
     if (!logits_old) return fail(OCC_ERR_INVALID_ARG, "null logits_old");

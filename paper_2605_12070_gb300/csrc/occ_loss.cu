@@ -150,7 +150,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_tma(const K2Args a) {
     }
     float lpo = 0.f, lpm = 0.f, A = 0.f;
     if (tid == 0) {
-      lpo = a.lp_old[row];
+      lpo = a.lp_old ? a.lp_old[row] : 0.f;
       lpm = a.lp_mu[row];
       A = a.adv[row];
     }
@@ -392,7 +392,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
     }
     float lpo = 0.f, lpm = 0.f, A = 0.f;
     if (tid == 0) {
-      lpo = a.lp_old[row];
+      lpo = a.lp_old ? a.lp_old[row] : 0.f;
       lpm = a.lp_mu[row];
       A = a.adv[row];
     }
@@ -591,7 +591,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
     float zy = 0.f, lpo = 0.f, lpm = 0.f, A = 0.f;
     if (tid == 0) {
       zy = Elem<Tin>::load(z + id);
-      lpo = a.lp_old[row];
+      lpo = a.lp_old ? a.lp_old[row] : 0.f;
       lpm = a.lp_mu[row];
       A = a.adv[row];
     }
@@ -714,7 +714,7 @@ __global__ void __launch_bounds__(NT) k2_loss_stream(const K2Args a) {
   float zy = 0.f, lpo = 0.f, lpm = 0.f, A = 0.f;
   if (tid == 0) {
     zy = Elem<Tin>::load(z + id);
-    lpo = a.lp_old[row];
+    lpo = a.lp_old ? a.lp_old[row] : 0.f;
     lpm = a.lp_mu[row];
     A = a.adv[row];
   }
@@ -973,8 +973,9 @@ extern "C" occ_status occ_decoupled_loss_fwd_bwd(
                                     logp_out, flags_out, dlogits, ld_grad, stats, workspace,
                                     ws_bytes, a, vec);
   if (st != OCC_OK) return st;
-  if (T > 0 && (!logp_old || !aligned(logp_old, 4)))
-    return fail(OCC_ERR_INVALID_ARG, "logp_old null or misaligned");
+  if (T > 0 && p->proxy == OCC_PROXY_NONE && !logp_old)
+    return fail(OCC_ERR_INVALID_ARG, "logp_old is null (and no proxy selected)");
+  if (logp_old && !aligned(logp_old, 4)) return fail(OCC_ERR_MISALIGNED, "logp_old misaligned");
   a.lp_old = logp_old;
   cudaStream_t s = (cudaStream_t)stream;
   st = launch_k0(a, s);

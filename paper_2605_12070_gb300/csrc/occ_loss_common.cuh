@@ -21,7 +21,22 @@ struct LossKParams {
   float grad_scale;
   int rd_weight;
   long long denom;                // > 0: caller's N; else read from the workspace
+  int proxy;                      // OCC_PROXY_*: how log pi_old is obtained
+  double alpha;                   // behaviour-policy weight of the proxy
 };
+
+// log pi_prox of a token from log mu_old and log pi_theta (Table 1 proxies,
+// App. A), in float64:
+//   log-linear:  alpha log mu + (1 - alpha) log pi_theta
+//   arithmetic:  log(alpha mu + (1 - alpha) pi_theta), written around the larger
+//                term as log1p of an expm1 so that it keeps relative precision.
+__device__ __forceinline__ double proxy_logprob(int proxy, double alpha, double lmu, double lth) {
+  if (proxy == OCC_PROXY_LOGLINEAR) return alpha * lmu + (1.0 - alpha) * lth;
+  const double d = lth - lmu;
+  if (d <= 0.0)  // mu >= pi_theta: alpha mu + (1-alpha) pi = mu (1 + (1-alpha) (e^d - 1))
+    return lmu + (double)log1pf((float)(1.0 - alpha) * expm1f((float)d));
+  return lth + (double)log1pf((float)alpha * expm1f((float)-d));
+}
 
 struct K2Args {
   const void* logits;
@@ -48,6 +63,7 @@ __device__ __forceinline__ void token_math(const LossKParams& kp, double lse, fl
                                            float lpm, float A, long long N, float& g,
                                            float& loss_t, uint32_t& flags, float& logp_f) {
   const double logp = (double)zy - lse;
+  if (kp.proxy != OCC_PROXY_NONE) lpo = proxy_logprob(kp.proxy, kp.alpha, (double)lpm, logp);
   const double log_rd = (double)lpo - (double)lpm;
   const bool in_band = (log_rd >= kp.log_rd_lo) && (log_rd <= kp.log_rd_hi);
   const double log_rs = logp - (double)lpo;
@@ -294,10 +310,13 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
                 (long long)T, (long long)V, (long long)ld);
   if (!(p->rd_lo >= 0.0) || !(p->rd_hi >= p->rd_lo) || !(p->eps_low >= 0.0) ||
       !(p->eps_low <= 1.0) || !(p->eps_high >= 0.0) || !isfinite(p->grad_scale) ||
-      (p->rd_weight != 0 && p->rd_weight != 1) || (p->dlogits_f32 != 0 && p->dlogits_f32 != 1))
+      (p->rd_weight != 0 && p->rd_weight != 1) || (p->dlogits_f32 != 0 && p->dlogits_f32 != 1) ||
+      p->proxy < OCC_PROXY_NONE || p->proxy > OCC_PROXY_ARITHMETIC ||
+      (p->proxy != OCC_PROXY_NONE && !(p->alpha >= 0.0 && p->alpha <= 1.0)))
     return fail(OCC_ERR_INVALID_ARG,
                 "thresholds must satisfy 0 <= rd_lo <= rd_hi, 0 <= eps_low <= 1, eps_high >= 0; "
-                "grad_scale finite; rd_weight and dlogits_f32 in {0,1}");
+                "grad_scale finite; rd_weight and dlogits_f32 in {0,1}; proxy in {0,1,2} with "
+                "alpha in [0,1]");
   if (!stats || !aligned(stats, 8)) return fail(OCC_ERR_INVALID_ARG, "stats null or misaligned");
   const WsLayout wl = ws_layout(T);
   if (!workspace || !aligned(workspace, 16) || ws_bytes < wl.total)
@@ -356,6 +375,8 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   a.kp.grad_scale = (float)p->grad_scale;
   a.kp.rd_weight = p->rd_weight;
   a.kp.denom = p->denom > 0 ? (long long)p->denom : 0;
+  a.kp.proxy = p->proxy;
+  a.kp.alpha = p->alpha;
   vec = T > 0 && aligned(logits, 16) && ((ld * (int64_t)es) % 16 == 0) &&
         (!dlogits || (aligned(dlogits, 16) && ((ld_grad * (int64_t)es_out) % 16 == 0)));
   return OCC_OK;

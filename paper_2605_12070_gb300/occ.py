@@ -45,7 +45,20 @@ class LossParams(ctypes.Structure):
     _fields_ = [("rd_lo", ctypes.c_double), ("rd_hi", ctypes.c_double),
                 ("eps_low", ctypes.c_double), ("eps_high", ctypes.c_double),
                 ("grad_scale", ctypes.c_double), ("denom", ctypes.c_int64),
-                ("rd_weight", ctypes.c_int32), ("dlogits_f32", ctypes.c_int32)]
+                ("rd_weight", ctypes.c_int32), ("dlogits_f32", ctypes.c_int32),
+                ("proxy", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("alpha", ctypes.c_double)]
+
+
+PROXY_NONE, PROXY_LOGLINEAR, PROXY_ARITHMETIC = 0, 1, 2
+_PROXIES = {None: 0, "none": 0, "loglinear": 1, "arithmetic": 2}
+
+
+def _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32,
+            proxy=None, alpha=0.0):
+    return LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
+                      float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)),
+                      _PROXIES[proxy], 0, float(alpha))
 
 
 _lib = None
@@ -179,11 +192,13 @@ def occ_decoupled_loss_fwd_bwd(logits, ids, logp_old, logp_mu, adv, loss_mask=No
                                rd_lo, rd_hi, eps_low, eps_high, rd_weight=1, grad_scale=1.0,
                                denom=0, dlogits_f32=False, dlogits="new", logp_out=None,
                                flags_out=None, want_logp=True, want_flags=True, stats=None,
-                               workspace=None, stream=None):
+                               workspace=None, stream=None, proxy=None, alpha=0.0):
     """The decoupled PPO loss over ``logits`` [T, V] and its gradient.
 
     ``dlogits``: "new" (allocate), None (forward only), "inplace" (overwrite
-    ``logits``), or a tensor [T, >=V].  Returns a dict with 'stats' (raw
+    ``logits``), or a tensor [T, >=V].  ``proxy`` ("loglinear" or "arithmetic",
+    with weight ``alpha``) builds log pi_old per token instead of reading
+    ``logp_old`` (which may then be None).  Returns a dict with 'stats' (raw
     device bytes), 'dlogits', 'logp', 'flags'.
     """
     _cuda(logits, ids, logp_old, logp_mu, adv, loss_mask)
@@ -210,8 +225,8 @@ def occ_decoupled_loss_fwd_bwd(logits, ids, logp_old, logp_mu, adv, loss_mask=No
         stats = new_loss_stats(dev)
     if workspace is None:
         workspace = new_workspace(T, V, dev)
-    p = LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
-                   float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)))
+    p = _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32,
+                proxy, alpha)
     rc = lib().occ_decoupled_loss_fwd_bwd(
         _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
         _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
@@ -262,8 +277,7 @@ def occ_decoupled_loss_fused(logits, logits_old, ids, logp_mu, adv, loss_mask=No
         stats = new_loss_stats(dev)
     if workspace is None:
         workspace = new_workspace(T, V, dev)
-    p = LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
-                   float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)))
+    p = _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32)
     rc = lib().occ_decoupled_loss_fused(
         _ptr(logits), _ptr(logits_old), _dtype_code(logits), T, V, ld, ld_old, _ptr(ids),
         _ptr(logp_mu), _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out),
@@ -291,8 +305,7 @@ def occ_decoupled_loss_fwd_bwd_noalloc(logits, ids, logp_old, logp_mu, adv, loss
     _cuda(logits, ids, logp_old, logp_mu, adv, loss_mask, dlogits, logp_out, flags_out, stats)
     T, V, ld = _rows(logits)
     ld_grad = dlogits.stride(0) if dlogits is not None else 0
-    p = LossParams(float(rd_lo), float(rd_hi), float(eps_low), float(eps_high),
-                   float(grad_scale), int(denom), int(rd_weight), int(bool(dlogits_f32)))
+    p = _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32)
     rc = lib().occ_decoupled_loss_fwd_bwd_noalloc(
         _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
         _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),

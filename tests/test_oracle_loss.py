@@ -21,7 +21,7 @@ import os
 import numpy as np
 import pytest
 
-from oracle import (LossParams, decoupled_loss, token_logprob, token_terms,
+from oracle import (LossParams, decoupled_loss, proxy_logprob, token_logprob, token_terms,
                     FLAG_ACTIVE, FLAG_CLIPPED, FLAG_IN_BAND, FLAG_VALID)
 
 P = LossParams(rd_lo=0.5, rd_hi=2.0, eps_low=0.2, eps_high=0.28)
@@ -152,12 +152,8 @@ def test_table4_effective_thresholds(golden_dir):
     lp_theta = lp_mu + np.log(r_theta)
     for (mlo, mhi, clo, chi, n, kind, e_mlo, e_mhi, e_clo, e_chi) in rows:
         alpha = 1.0 / (n + 1)
-        if kind == "loglinear":
-            # log pi_prox = alpha log mu_old + (1 - alpha) log pi_theta
-            lp_prox = alpha * lp_mu + (1 - alpha) * lp_theta
-        else:
-            # pi_prox = alpha mu_old + (1 - alpha) pi_theta
-            lp_prox = np.log(alpha * np.exp(lp_mu) + (1 - alpha) * np.exp(lp_theta))
+        # Table 4's "Linear" rows are the arithmetic proxy (linear_prox of Table 1)
+        lp_prox = proxy_logprob({"linear": "arithmetic"}.get(kind, kind), alpha, lp_mu, lp_theta)
         p = LossParams(mlo, mhi, 1.0 - clo, chi - 1.0)
         for A, which in ((1.0, "hi"), (-1.0, "lo")):
             out = token_terms(lp_theta, lp_prox, lp_mu, np.full(r_theta.size, A), None, p)
@@ -289,3 +285,26 @@ def test_caller_denominator_and_grad_scale():
     out = decoupled_loss(z, ids, lp_old, lp_mu, adv, None, p2)
     assert abs(out["loss"] * 80 - base["loss"] * 20) < 1e-13
     np.testing.assert_allclose(out["dlogits"] * 80 / 3.0, base["dlogits"] * 20, atol=1e-15)
+
+
+def test_proxy_ratio_closed_forms():
+    """App. A: with the log-linear proxy r_d = r^(1-alpha) and r_s = r^alpha; with
+    the arithmetic proxy r_d = alpha + (1 - alpha) r, where r = pi_theta / mu_old."""
+    rng = np.random.default_rng(80)
+    lmu = rng.normal(-4, 1, size=50)
+    r = np.exp(rng.normal(0, 0.3, size=50))
+    lth = lmu + np.log(r)
+    for alpha in (0.25, 1 / 3, 0.5, 0.9):
+        for kind in ("loglinear", "arithmetic"):
+            lp = proxy_logprob(kind, alpha, lmu, lth)
+            out = token_terms(lth, lp, lmu, np.ones(50), None, P)
+            if kind == "loglinear":
+                np.testing.assert_allclose(out["r_d"], r ** (1 - alpha), rtol=1e-12)
+                np.testing.assert_allclose(out["r_s"], r ** alpha, rtol=1e-12)
+            else:
+                np.testing.assert_allclose(out["r_d"], alpha + (1 - alpha) * r, rtol=1e-12)
+                np.testing.assert_allclose(out["r_s"], r / (alpha + (1 - alpha) * r), rtol=1e-12)
+    # alpha = 0 gives pi_prox = pi_theta (r_s = 1); alpha = 1 gives mu_old (r_d = 1)
+    for kind in ("loglinear", "arithmetic"):
+        np.testing.assert_allclose(proxy_logprob(kind, 0.0, lmu, lth), lth, atol=1e-13)
+        np.testing.assert_allclose(proxy_logprob(kind, 1.0, lmu, lth), lmu, atol=1e-13)
