@@ -259,6 +259,48 @@ occ_status occ_ewma_update(float* theta_prox, const float* theta, int64_t n, dou
                            occ_ewma_state* st, const occ_loss_stats* stats, double tau,
                            int32_t min_streak, int32_t force_reset, void* stream);
 
+/*
+ * occ_ewma_update_bf16 -- occ_ewma_update with the proximal parameters stored
+ * in bf16 (2 bytes per parameter, the footprint of the paper's host-side EWMA
+ * copy, Table 3a).
+ *
+ * Same coefficients, reset rule and state as occ_ewma_update.  Each parameter
+ * is updated in float32 from its bf16 value, v = tp + b (theta - tp), and
+ * rounded back to bf16: to nearest-even when sr_seed == 0, else
+ * stochastically -- 16 random bits, the i-th output of the SplitMix64
+ * generator started at sr_seed (i = the parameter index), are added below the
+ * bf16 unit in the last place before truncation, so an EWMA step smaller than
+ * half a bf16 ulp is kept in expectation.  Pass a different seed per step.
+ *
+ *   theta_prox [n] bf16, updated in place;  theta [n] float32 or bf16 (theta_dt)
+ */
+occ_status occ_ewma_update_bf16(void* theta_prox, const void* theta, occ_dtype theta_dt,
+                                int64_t n, double beta, occ_ewma_state* st,
+                                const occ_loss_stats* stats, double tau, int32_t min_streak,
+                                int32_t force_reset, uint64_t sr_seed, void* stream);
+
+/*
+ * occ_ewma_update_host -- the PPO-EWMA step with the proximal parameters kept
+ * in PINNED HOST memory (where the paper keeps its EWMA copy, Table 3a),
+ * streamed through the GPU.
+ *
+ * theta_prox_host (float32 or bf16, prox_dt) is copied in chunks into two
+ * slots of the caller's device `staging` buffer, updated there (the
+ * occ_ewma_update / occ_ewma_update_bf16 arithmetic; theta [n] is on the
+ * device) and copied back, alternating stream0 and stream1 so that copies in
+ * both directions overlap the updates.  The coefficient step runs once, on
+ * stream0; the call's work is complete when stream0 reaches the point of the
+ * call (stream1 is joined back into stream0).  A float32 buffer needs float32
+ * theta.  staging_bytes sets the chunk size (two slots; at least 2 x 16 bytes
+ * of elements); theta_prox_host and staging are 16-byte aligned.  Returns
+ * OCC_ERR_INVALID_ARG if theta_prox_host is not page-locked.
+ */
+occ_status occ_ewma_update_host(void* theta_prox_host, occ_dtype prox_dt, const void* theta,
+                                occ_dtype theta_dt, int64_t n, double beta, occ_ewma_state* st,
+                                const occ_loss_stats* stats, double tau, int32_t min_streak,
+                                int32_t force_reset, uint64_t sr_seed, void* staging,
+                                size_t staging_bytes, void* stream0, void* stream1);
+
 /* Sets a DEVICE occ_ewma_state to {w = w0, streak = 0, n_resets = 0}: w0 = 0 for an
  * empty history, 1/(1-beta) to start in the stationary regime. */
 occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* stream);

@@ -38,4 +38,5 @@ from .loss import LossParams, token_logprob, token_terms, decoupled_loss, softma
 from .diagnostics import token_entropy, token_kl  # noqa: F401
 from .proxies import proxy_logprob  # noqa: F401
 from .ewma import EwmaState, ewma_coefficients, ewma_update, ewma_closed_form, \
-    beta_for_window, center_of_mass  # noqa: F401
+    beta_for_window, center_of_mass, splitmix64_at, round_bf16, bf16_bits_to_f32, \
+    ewma_update_bf16  # noqa: F401

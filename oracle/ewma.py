@@ -16,6 +16,9 @@ below tau.  App. D speaks of consecutive low-ratio streaks; the oracle counts
 a streak and resets once it reaches ``min_streak`` (1 = reset on the first low
 step, the Sec. 5.2 rule).  A step with no valid tokens carries no evidence:
 the streak is left unchanged.
+
+A bf16 proximal buffer (the footprint of the paper's host-side copy, Table 3a)
+is modelled in the kernel's precision, see ``ewma_update_bf16``.
 """
 
 from dataclasses import dataclass, replace
@@ -81,3 +84,75 @@ def beta_for_window(W):
 def center_of_mass(beta):
     """App. B: stationary center of mass of the EWMA history, beta / (1 - beta)."""
     return beta / (1.0 - beta)
+
+
+# --------------------------------------------------------------- bf16 buffers
+#
+# For a bf16 proximal buffer the stored value is a quantised code, so the
+# oracle takes the rounding decision in the kernel's precision: the update is
+# formed in float32 (one rounding of theta - theta_prox, one fused
+# multiply-add), then rounded to bf16 by definition: nearest with ties to even,
+# or stochastically with the bits of a SplitMix64 counter stream.
+
+_GAMMA = np.uint64(0x9E3779B97F4A7C15)
+
+
+def splitmix64_at(seed, i):
+    """The i-th output (i >= 0) of SplitMix64 started at `seed` (Steele, Lea and
+    Flood, 2014): state_i = seed + (i + 1) gamma, output = mix(state_i)."""
+    with np.errstate(over="ignore"):
+        z = np.uint64(seed) + (np.asarray(i, dtype=np.uint64) + np.uint64(1)) * _GAMMA
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
+        return z ^ (z >> np.uint64(31))
+
+
+def bf16_bits_to_f32(bits):
+    return (np.asarray(bits, dtype=np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def round_bf16(x32, seed=0, idx=None):
+    """float32 -> bf16 bits.  seed == 0: nearest, ties to even.  Otherwise add the
+    top 16 bits of the generator output below the bf16 unit in the last place
+    and truncate (stochastic rounding of the magnitude)."""
+    u = np.asarray(x32, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    special = (u & np.uint64(0x7F800000)) == np.uint64(0x7F800000)
+    if seed == 0:
+        lsb = (u >> np.uint64(16)) & np.uint64(1)
+        r = np.uint64(0x7FFF) + lsb
+    else:
+        r = splitmix64_at(seed, idx) >> np.uint64(48)
+    out = ((u + r) >> np.uint64(16)) & np.uint64(0xFFFF)
+    trunc = (u >> np.uint64(16)) & np.uint64(0xFFFF)
+    return np.where(special, trunc, out).astype(np.uint16)
+
+
+def fma_f32(a, b, c):
+    """float32 fused multiply-add a * b + c, rounded once to nearest-even.
+
+    The product of two float32 values is exact in float64; the float64 sum is
+    exact up to its TwoSum error e.  Rounding s = fl64(p + c) to float32 is
+    then correct except when s falls exactly on a float32 midpoint, where the
+    sign of e decides the side."""
+    p = np.asarray(a, np.float64) * np.asarray(b, np.float64)
+    c = np.asarray(c, np.float64)
+    s = p + c
+    bp = s - p
+    e = (p - (s - bp)) + (c - bp)                  # TwoSum: p + c = s + e exactly
+    r = s.astype(np.float32)
+    d = s - r.astype(np.float64)                   # exact
+    half = np.spacing(np.abs(r)).astype(np.float64) / 2
+    fix = (np.abs(d) == half) & (d * e > 0)        # past the midpoint: round away from r
+    r = np.where(fix, np.nextafter(r, np.where(d > 0, np.float32(np.inf), np.float32(-np.inf))), r)
+    return r.astype(np.float32)
+
+
+def ewma_update_bf16(tp_bits, theta32, b, copy, seed=0, idx0=0):
+    """One App. B step on a bf16 buffer in the kernel's precision:
+    v = fma(b, theta - tp, tp) in float32 (or theta itself on a reset / first
+    step), rounded to bf16."""
+    tp = bf16_bits_to_f32(tp_bits)
+    th = np.asarray(theta32, dtype=np.float32)
+    v = th if copy else fma_f32(np.float32(b), (th - tp).astype(np.float32), tp)
+    idx = np.arange(idx0, idx0 + tp.size, dtype=np.uint64)
+    return round_bf16(v, seed, idx)

@@ -10,6 +10,8 @@
 // theta bit for bit.  HBM traffic: 12 bytes per parameter (two reads, one write).
 #include "occ_common.cuh"
 
+#include <algorithm>
+
 namespace occ {
 
 constexpr int kK3Threads = 256;
@@ -118,6 +120,95 @@ __global__ void k3_state_init(occ_ewma_state* st, double w0) {
   st->reserved = 0;
 }
 
+
+// ------------------------------------------------------------------ bf16 buffers
+//
+// The proximal parameters may be kept in bf16 (2 bytes per parameter, the
+// footprint the paper reports for its host-side EWMA copy, Table 3a).  The
+// update is computed in float32 from the bf16 value and rounded back either
+// to nearest-even or stochastically (seed != 0), which keeps small EWMA steps
+// (b (theta - theta_prox) below half a bf16 ulp) from being lost in
+// expectation.
+
+// The i-th output of SplitMix64 (Steele, Lea and Flood, 2014) started at
+// `seed`, used as a counter-based generator: state_i = seed + (i + 1) gamma.
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t i) {
+  uint64_t z = seed + (i + 1) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// float32 -> bf16 bits: nearest-even (seed == 0) or stochastic: 16 random bits
+// are added below the bf16 unit in the last place and the result truncated,
+// so the magnitude rounds up with probability equal to the dropped fraction.
+__device__ __forceinline__ uint16_t round_bf16(float x, uint64_t seed, uint64_t idx) {
+  const uint32_t u = __float_as_uint(x);
+  if (seed == 0 || (u & 0x7f800000u) == 0x7f800000u) {
+    unsigned short h;
+    asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(x));
+    return h;
+  }
+  const uint32_t r = (uint32_t)(splitmix64_at(seed, idx) >> 48);
+  return (uint16_t)((u + r) >> 16);
+}
+
+template <typename ThT>
+__device__ __forceinline__ void load8(const ThT* p, float (&x)[8]);
+template <>
+__device__ __forceinline__ void load8<float>(const float* p, float (&x)[8]) {
+  const uint4 a = ld_stream_v4(p), b = ld_stream_v4(p + 4);
+  x[0] = __uint_as_float(a.x); x[1] = __uint_as_float(a.y);
+  x[2] = __uint_as_float(a.z); x[3] = __uint_as_float(a.w);
+  x[4] = __uint_as_float(b.x); x[5] = __uint_as_float(b.y);
+  x[6] = __uint_as_float(b.z); x[7] = __uint_as_float(b.w);
+}
+template <>
+__device__ __forceinline__ void load8<bf16_t>(const bf16_t* p, float (&x)[8]) {
+  Elem<bf16_t>::unpack(ld_stream_v4(p), x);
+}
+__device__ __forceinline__ float load1(const float* p) { return *p; }
+__device__ __forceinline__ float load1(const bf16_t* p) {
+  return __uint_as_float(((uint32_t)p->bits) << 16);
+}
+
+// theta_prox (bf16, 16-byte aligned) <- theta_prox + b (theta - theta_prox),
+// eight parameters per thread iteration; elements [8 n8, n) in a scalar tail.
+template <typename ThT, int NT>
+__global__ void __launch_bounds__(NT) k3_ewma_bf16(bf16_t* __restrict__ tp,
+                                                   const ThT* __restrict__ th, int64_t n,
+                                                   bool vec, const occ_ewma_state* __restrict__ st,
+                                                   uint64_t seed, uint64_t idx0) {
+  const double bd = st->coef_b;
+  const bool copy = (bd == 1.0);
+  const float b = (float)bd;
+  const int64_t stride = (int64_t)gridDim.x * NT;
+  const int64_t gtid = (int64_t)blockIdx.x * NT + threadIdx.x;
+  int64_t done = 0;
+  if (vec) {
+    const int64_t n8 = n / 8;
+    for (int64_t i = gtid; i < n8; i += stride) {
+      float x[8], y[8];
+      Elem<bf16_t>::unpack(ld_stream_v4(tp + 8 * i), x);
+      load8<ThT>(th + 8 * i, y);
+      uint16_t o[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float v = copy ? y[k] : fmaf(b, y[k] - x[k], x[k]);
+        o[k] = round_bf16(v, seed, idx0 + 8 * i + k);
+      }
+      st_stream_v4(tp + 8 * i, make_uint4(o[0] | ((uint32_t)o[1] << 16), o[2] | ((uint32_t)o[3] << 16),
+                                          o[4] | ((uint32_t)o[5] << 16), o[6] | ((uint32_t)o[7] << 16)));
+    }
+    done = n8 * 8;
+  }
+  for (int64_t i = done + gtid; i < n; i += stride) {
+    const float x = load1(tp + i), y = load1(th + i);
+    const float v = copy ? y : fmaf(b, y - x, x);
+    tp[i].bits = round_bf16(v, seed, idx0 + i);
+  }
+}
+
 }  // namespace occ
 
 using namespace occ;
@@ -169,4 +260,152 @@ extern "C" occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* s
   if (!(w0 >= 0.0) || isinf(w0)) return fail(OCC_ERR_INVALID_ARG, "w0 must be finite and >= 0");
   k3_state_init<<<1, 1, 0, (cudaStream_t)stream>>>(st, w0);
   return check_launch("occ_ewma_state_init");
+}
+
+
+// ------------------------------------------------------------------ F4 entry points
+
+namespace {
+
+occ_status validate_ewma(int64_t n, double beta, occ_ewma_state* st, const occ_loss_stats* stats,
+                         double tau, int32_t min_streak) {
+  if (n < 0) return fail(OCC_ERR_INVALID_ARG, "n < 0");
+  if (!st || !aligned(st, 8)) return fail(OCC_ERR_INVALID_ARG, "state null or misaligned");
+  if (stats && !aligned(stats, 8)) return fail(OCC_ERR_MISALIGNED, "stats misaligned");
+  if (!(beta >= 0.0 && beta < 1.0)) return fail(OCC_ERR_INVALID_ARG, "beta must be in [0, 1)");
+  if (min_streak < 1) return fail(OCC_ERR_INVALID_ARG, "min_streak must be >= 1");
+  if (isnan(tau)) return fail(OCC_ERR_INVALID_ARG, "tau is NaN");
+  return OCC_OK;
+}
+
+// Launches the bf16 update of n parameters whose global index starts at idx0.
+occ_status launch_bf16_body(bf16_t* tp, const void* th, occ_dtype theta_dt, int64_t n,
+                            const occ_ewma_state* st, uint64_t seed, uint64_t idx0,
+                            cudaStream_t s) {
+  if (n == 0) return OCC_OK;
+  const bool vec = aligned(tp, 16) && aligned(th, 16);
+  const int64_t work = vec ? (n + 7) / 8 : n;
+  const int64_t need = (work + kK3Threads - 1) / kK3Threads;
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, (int64_t)sm_count() * 8));
+  if (theta_dt == OCC_BF16)
+    k3_ewma_bf16<bf16_t, kK3Threads><<<grid, kK3Threads, 0, s>>>(tp, (const bf16_t*)th, n, vec, st,
+                                                                 seed, idx0);
+  else
+    k3_ewma_bf16<float, kK3Threads><<<grid, kK3Threads, 0, s>>>(tp, (const float*)th, n, vec, st,
+                                                                seed, idx0);
+  return check_launch("k3_ewma_bf16");
+}
+
+// Launches the float32 update of n parameters (vector body + scalar tail).
+occ_status launch_f32_body(float* tp, const float* th, int64_t n, const occ_ewma_state* st,
+                           cudaStream_t s) {
+  if (n == 0) return OCC_OK;
+  const int64_t blocks_cap = (int64_t)sm_count() * 8;
+  if (aligned(tp, 16) && aligned(th, 16)) {
+    const int64_t n4 = n / 4;
+    if (n4 > 0) {
+      const int64_t need = (n4 + kK3Threads * kK3Unroll - 1) / (kK3Threads * kK3Unroll);
+      const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
+      k3_ewma_vec<kK3Threads, kK3Unroll><<<grid, kK3Threads, 0, s>>>((float4*)tp,
+                                                                     (const float4*)th, n4, st);
+    }
+    if (n - n4 * 4 > 0) k3_ewma_scalar<kK3Threads><<<1, kK3Threads, 0, s>>>(tp, th, n4 * 4, n, st);
+  } else {
+    const int64_t need = (n + kK3Threads - 1) / kK3Threads;
+    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
+    k3_ewma_scalar<kK3Threads><<<grid, kK3Threads, 0, s>>>(tp, th, 0, n, st);
+  }
+  return check_launch("k3_ewma body");
+}
+
+}  // namespace
+
+extern "C" occ_status occ_ewma_update_bf16(void* theta_prox, const void* theta, occ_dtype theta_dt,
+                                           int64_t n, double beta, occ_ewma_state* st,
+                                           const occ_loss_stats* stats, double tau,
+                                           int32_t min_streak, int32_t force_reset,
+                                           uint64_t sr_seed, void* stream) {
+  clear_error();
+  occ_status rc = validate_ewma(n, beta, st, stats, tau, min_streak);
+  if (rc != OCC_OK) return rc;
+  if (theta_dt != OCC_F32 && theta_dt != OCC_BF16)
+    return fail(OCC_ERR_UNSUPPORTED, "theta dtype %d", (int)theta_dt);
+  const size_t es = dtype_size(theta_dt);
+  if (n > 0) {
+    if (!theta_prox || !theta) return fail(OCC_ERR_INVALID_ARG, "null theta_prox/theta");
+    if (!aligned(theta_prox, 2) || !aligned(theta, es))
+      return fail(OCC_ERR_MISALIGNED, "arrays must be aligned to their element size");
+    if (overlaps(theta_prox, (size_t)n * 2, theta, (size_t)n * es))
+      return fail(OCC_ERR_INVALID_ARG, "theta_prox overlaps theta");
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  k3_ewma_prologue<<<1, 1, 0, s>>>(st, stats, beta, tau, min_streak, force_reset ? 1 : 0);
+  rc = check_launch("k3_ewma_prologue");
+  if (rc != OCC_OK) return rc;
+  return launch_bf16_body((bf16_t*)theta_prox, theta, theta_dt, n, st, sr_seed, 0, s);
+}
+
+extern "C" occ_status occ_ewma_update_host(void* theta_prox_host, occ_dtype prox_dt,
+                                           const void* theta, occ_dtype theta_dt, int64_t n,
+                                           double beta, occ_ewma_state* st,
+                                           const occ_loss_stats* stats, double tau,
+                                           int32_t min_streak, int32_t force_reset,
+                                           uint64_t sr_seed, void* staging, size_t staging_bytes,
+                                           void* stream0, void* stream1) {
+  clear_error();
+  occ_status rc = validate_ewma(n, beta, st, stats, tau, min_streak);
+  if (rc != OCC_OK) return rc;
+  if ((prox_dt != OCC_F32 && prox_dt != OCC_BF16) || (theta_dt != OCC_F32 && theta_dt != OCC_BF16))
+    return fail(OCC_ERR_UNSUPPORTED, "dtypes %d/%d", (int)prox_dt, (int)theta_dt);
+  if (prox_dt == OCC_F32 && theta_dt != OCC_F32)
+    return fail(OCC_ERR_UNSUPPORTED, "a float32 proximal buffer needs float32 theta");
+  const size_t pes = dtype_size(prox_dt), tes = dtype_size(theta_dt);
+  if (n > 0) {
+    if (!theta_prox_host || !theta || !staging)
+      return fail(OCC_ERR_INVALID_ARG, "null theta_prox_host/theta/staging");
+    if (!aligned(theta_prox_host, 16) || !aligned(staging, 16) || !aligned(theta, tes))
+      return fail(OCC_ERR_MISALIGNED, "host buffer and staging must be 16-byte aligned");
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, theta_prox_host) != cudaSuccess ||
+        at.type != cudaMemoryTypeHost) {
+      cudaGetLastError();
+      return fail(OCC_ERR_INVALID_ARG, "theta_prox_host must be pinned (page-locked) host memory");
+    }
+  }
+  // two staging slots, each a whole number of 16-byte groups
+  const int64_t chunk = (int64_t)(staging_bytes / 2 / pes) / 8 * 8;
+  if (n > 0 && chunk <= 0)
+    return fail(OCC_ERR_WORKSPACE, "staging needs at least %zu bytes", 2 * 8 * pes);
+  cudaStream_t s[2] = {(cudaStream_t)stream0, (cudaStream_t)stream1};
+  k3_ewma_prologue<<<1, 1, 0, s[0]>>>(st, stats, beta, tau, min_streak, force_reset ? 1 : 0);
+  rc = check_launch("k3_ewma_prologue");
+  if (rc != OCC_OK || n == 0) return rc;
+  cudaEvent_t ev;
+  if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess)
+    return check_launch("cudaEventCreate");
+  if (s[1] != s[0]) {  // stream 1 starts after the coefficients exist
+    cudaEventRecord(ev, s[0]);
+    cudaStreamWaitEvent(s[1], ev, 0);
+  }
+  char* host = (char*)theta_prox_host;
+  char* stage[2] = {(char*)staging, (char*)staging + (size_t)chunk * pes};
+  for (int64_t k = 0, off = 0; off < n; ++k, off += chunk) {
+    const int64_t m = std::min(chunk, n - off);
+    cudaStream_t q = s[k & 1];
+    char* buf = stage[k & 1];
+    cudaMemcpyAsync(buf, host + (size_t)off * pes, (size_t)m * pes, cudaMemcpyHostToDevice, q);
+    const void* th = (const char*)theta + (size_t)off * tes;
+    rc = prox_dt == OCC_F32
+             ? launch_f32_body((float*)buf, (const float*)th, m, st, q)
+             : launch_bf16_body((bf16_t*)buf, th, theta_dt, m, st, sr_seed, (uint64_t)off, q);
+    if (rc != OCC_OK) break;
+    cudaMemcpyAsync(host + (size_t)off * pes, buf, (size_t)m * pes, cudaMemcpyDeviceToHost, q);
+  }
+  if (s[1] != s[0]) {  // the call completes on stream 0
+    cudaEventRecord(ev, s[1]);
+    cudaStreamWaitEvent(s[0], ev, 0);
+  }
+  cudaEventDestroy(ev);
+  if (rc != OCC_OK) return rc;
+  return check_launch("occ_ewma_update_host");
 }

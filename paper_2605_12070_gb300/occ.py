@@ -32,7 +32,8 @@ _STATE_FMT = "<3d4i"
 
 # Every symbol declared in include/occ.h.
 EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_fwd_bwd",
-           "occ_decoupled_loss_fused", "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update", "occ_ewma_state_init",
+           "occ_decoupled_loss_fused", "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update",
+           "occ_ewma_update_bf16", "occ_ewma_update_host", "occ_ewma_state_init",
            "occ_status_string", "occ_last_error", "occ_version")
 
 
@@ -92,6 +93,12 @@ def lib():
     L.occ_decoupled_loss_fwd_bwd_noalloc.restype = i32
     L.occ_ewma_update.argtypes = [vp, vp, i64, dbl, vp, vp, dbl, i32, i32, vp]
     L.occ_ewma_update.restype = i32
+    u64 = ctypes.c_uint64
+    L.occ_ewma_update_bf16.argtypes = [vp, vp, i32, i64, dbl, vp, vp, dbl, i32, i32, u64, vp]
+    L.occ_ewma_update_bf16.restype = i32
+    L.occ_ewma_update_host.argtypes = [vp, i32, vp, i32, i64, dbl, vp, vp, dbl, i32, i32, u64, vp,
+                                       ctypes.c_size_t, vp, vp]
+    L.occ_ewma_update_host.restype = i32
     L.occ_ewma_state_init.argtypes = [vp, dbl, vp]
     L.occ_ewma_state_init.restype = i32
     L.occ_status_string.argtypes = [i32]
@@ -357,3 +364,46 @@ def occ_ewma_update(theta_prox, theta, beta, state, stats=None, tau=0.9, min_str
                                _stream(stream, theta_prox.device))
     _check(rc, "occ_ewma_update")
     return theta_prox
+
+
+def _float_code(t):
+    if t.dtype == torch.bfloat16:
+        return OCC_BF16
+    if t.dtype == torch.float32:
+        return OCC_F32
+    raise OccError(f"unsupported dtype {t.dtype}")
+
+
+def occ_ewma_update_bf16(theta_prox, theta, beta, state, stats=None, tau=0.9, min_streak=1,
+                         force_reset=False, sr_seed=0, stream=None):
+    """PPO-EWMA step on a bf16 proximal buffer (theta float32 or bf16); sr_seed != 0
+    selects stochastic rounding."""
+    _cuda(theta_prox, theta, state, stats)
+    if theta_prox.dtype != torch.bfloat16 or not theta_prox.is_contiguous() or \
+            not theta.is_contiguous() or theta.numel() != theta_prox.numel():
+        raise OccError("theta_prox must be contiguous bf16 and match theta")
+    rc = lib().occ_ewma_update_bf16(_ptr(theta_prox), _ptr(theta), _float_code(theta),
+                                    theta_prox.numel(), float(beta), _ptr(state), _ptr(stats),
+                                    float(tau), int(min_streak), int(bool(force_reset)),
+                                    int(sr_seed), _stream(stream, theta_prox.device))
+    _check(rc, "occ_ewma_update_bf16")
+    return theta_prox
+
+
+def occ_ewma_update_host(theta_prox_host, theta, beta, state, staging, stats=None, tau=0.9,
+                         min_streak=1, force_reset=False, sr_seed=0, stream0=None, stream1=None):
+    """PPO-EWMA step on a pinned host proximal buffer, streamed through ``staging``
+    (a device uint8 tensor) on two streams."""
+    _cuda(theta, state, stats, staging)
+    if theta_prox_host.is_cuda or not theta_prox_host.is_pinned():
+        raise OccError("theta_prox_host must be a pinned host tensor")
+    dev = theta.device
+    s0 = stream0 if stream0 is not None else torch.cuda.current_stream(dev)
+    s1 = stream1 if stream1 is not None else s0
+    rc = lib().occ_ewma_update_host(
+        _ptr(theta_prox_host), _float_code(theta_prox_host), _ptr(theta), _float_code(theta),
+        theta.numel(), float(beta), _ptr(state), _ptr(stats), float(tau), int(min_streak),
+        int(bool(force_reset)), int(sr_seed), _ptr(staging), staging.numel(),
+        ctypes.c_void_p(s0.cuda_stream), ctypes.c_void_p(s1.cuda_stream))
+    _check(rc, "occ_ewma_update_host")
+    return theta_prox_host

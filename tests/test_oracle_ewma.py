@@ -91,3 +91,74 @@ def test_streak_rule():
     assert resets == [(False, 1), (False, 0), (False, 1), (True, 0), (False, 0), (False, 1)]
     _, _, reset, _ = ewma_coefficients(EwmaState(w=2.0), 0.75, force_reset=True)
     assert reset
+
+
+# ---------------------------------------------------------------- bf16 buffers
+
+def test_splitmix64_reference_outputs():
+    # Reference outputs of SplitMix64 for seed 1234567, as printed by its public
+    # reference implementation (Steele, Lea and Flood 2014; splitmix64.c).
+    from oracle import splitmix64_at
+    expect = [6457827717110365317, 3203168211198807973, 9817491932198370423,
+              4593380528125082431, 16408922859458223821]
+    assert [int(v) for v in splitmix64_at(1234567, np.arange(5))] == expect
+
+
+def test_bf16_nearest_matches_torch_and_ties_to_even():
+    torch = pytest.importorskip("torch")
+    from oracle import round_bf16
+    rng = np.random.default_rng(3)
+    x = (rng.standard_normal(100000) * np.exp(rng.uniform(-20, 20, 100000))).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(round_bf16(x), ref)
+    # exact midpoints: 1 + 2^-8 lies between 1 and 1 + 2^-7 -> even (1.0)
+    mid = np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8], dtype=np.float32)
+    out = round_bf16(mid)
+    assert out[0] == 0x3F80 and out[1] == 0x3F82
+
+
+def test_bf16_stochastic_rounding_is_unbiased_and_brackets():
+    from oracle import bf16_bits_to_f32, round_bf16
+    x = np.full(200000, 1.0 + 0.3 * 2.0 ** -7, dtype=np.float32)   # 30 % of a bf16 ulp above 1
+    bits = round_bf16(x, seed=99, idx=np.arange(x.size, dtype=np.uint64))
+    vals = bf16_bits_to_f32(bits)
+    assert set(np.unique(vals).tolist()) == {1.0, 1.0 + 2.0 ** -7}
+    frac = np.mean(vals > 1.0)
+    assert abs(frac - 0.3) < 0.005                      # rounds up with the dropped fraction
+    assert abs(vals.astype(np.float64).mean() - float(x[0])) < 2e-5
+    neg = round_bf16(-x, seed=99, idx=np.arange(x.size, dtype=np.uint64))
+    assert np.array_equal(neg, bits | 0x8000)          # magnitude rounding: sign symmetric
+
+
+def test_bf16_step_tracks_float64_recursion():
+    from oracle import bf16_bits_to_f32, ewma_update_bf16, round_bf16
+    rng = np.random.default_rng(4)
+    th = (rng.standard_normal(50000) * 0.02).astype(np.float32)
+    tp = round_bf16((th + rng.standard_normal(50000) * 1e-3).astype(np.float32))
+    exact = 0.25 * bf16_bits_to_f32(tp).astype(np.float64) + 0.75 * th
+    out = bf16_bits_to_f32(ewma_update_bf16(tp, th, 0.75, copy=False)).astype(np.float64)
+    ulp = np.abs(exact) * 2.0 ** -7
+    assert np.all(np.abs(out - exact) <= 0.5 * ulp * (1 + 1e-3) + 1e-12)
+    assert np.array_equal(ewma_update_bf16(tp, th, 1.0, copy=True), round_bf16(th))
+
+
+def test_fma_f32_single_rounding():
+    from fractions import Fraction
+    from oracle.ewma import fma_f32
+    rng = np.random.default_rng(5)
+    a = rng.standard_normal(2000).astype(np.float32)
+    b = (rng.standard_normal(2000) * 1e-3).astype(np.float32)
+    c = rng.standard_normal(2000).astype(np.float32)
+    # midpoint constructions: c + a*b lands exactly half a float32 ulp plus a tiny product
+    c[:8] = np.float32(1.0)
+    a[:8] = np.float32(2.0 ** -24)
+    b[:8] = np.float32(1.0) + np.float32(2.0 ** -23) * np.arange(8, dtype=np.float32)
+    got = fma_f32(a, b, c)
+    for i in range(2000):
+        exact = Fraction(float(a[i])) * Fraction(float(b[i])) + Fraction(float(c[i]))
+        lo = np.float32(float(exact))
+        # correctly rounded float32 of the exact value: compare against both neighbours
+        cands = [lo, np.nextafter(lo, np.float32(np.inf)), np.nextafter(lo, np.float32(-np.inf))]
+        best = min(cands, key=lambda x: (abs(Fraction(float(x)) - exact),
+                                        int(np.float32(x).view(np.uint32)) & 1))
+        assert got[i] == best, i
