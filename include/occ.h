@@ -267,10 +267,11 @@ occ_status occ_ewma_update(float* theta_prox, const float* theta, int64_t n, dou
  * Same coefficients, reset rule and state as occ_ewma_update.  Each parameter
  * is updated in float32 from its bf16 value, v = tp + b (theta - tp), and
  * rounded back to bf16: to nearest-even when sr_seed == 0, else
- * stochastically -- 16 random bits, the i-th output of the SplitMix64
- * generator started at sr_seed (i = the parameter index), are added below the
- * bf16 unit in the last place before truncation, so an EWMA step smaller than
- * half a bf16 ulp is kept in expectation.  Pass a different seed per step.
+ * stochastically -- 16 random bits are added below the bf16 unit in the last
+ * place before truncation, so an EWMA step smaller than half a bf16 ulp is
+ * kept in expectation.  Parameter i takes 16-bit lane (i mod 4), least
+ * significant first, of the (i / 4)-th output of the SplitMix64 generator
+ * started at sr_seed.  Pass a different seed per step.
  *
  *   theta_prox [n] bf16, updated in place;  theta [n] float32 or bf16 (theta_dt)
  */

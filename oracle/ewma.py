@@ -111,17 +111,25 @@ def bf16_bits_to_f32(bits):
     return (np.asarray(bits, dtype=np.uint32) << np.uint32(16)).view(np.float32)
 
 
+def sr_bits(seed, idx):
+    """16 random bits for parameter idx: lane (idx mod 4) of the (idx // 4)-th
+    SplitMix64 output, lane 0 being the least significant 16 bits."""
+    idx = np.asarray(idx, dtype=np.uint64)
+    out = splitmix64_at(seed, idx >> np.uint64(2))
+    return (out >> (np.uint64(16) * (idx & np.uint64(3)))) & np.uint64(0xFFFF)
+
+
 def round_bf16(x32, seed=0, idx=None):
-    """float32 -> bf16 bits.  seed == 0: nearest, ties to even.  Otherwise add the
-    top 16 bits of the generator output below the bf16 unit in the last place
-    and truncate (stochastic rounding of the magnitude)."""
+    """float32 -> bf16 bits.  seed == 0: nearest, ties to even.  Otherwise add 16
+    random bits (``sr_bits``) below the bf16 unit in the last place and
+    truncate (stochastic rounding of the magnitude)."""
     u = np.asarray(x32, dtype=np.float32).view(np.uint32).astype(np.uint64)
     special = (u & np.uint64(0x7F800000)) == np.uint64(0x7F800000)
     if seed == 0:
         lsb = (u >> np.uint64(16)) & np.uint64(1)
         r = np.uint64(0x7FFF) + lsb
     else:
-        r = splitmix64_at(seed, idx) >> np.uint64(48)
+        r = sr_bits(seed, idx)
     out = ((u + r) >> np.uint64(16)) & np.uint64(0xFFFF)
     trunc = (u >> np.uint64(16)) & np.uint64(0xFFFF)
     return np.where(special, trunc, out).astype(np.uint16)

@@ -139,18 +139,24 @@ __device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t i) {
   return z ^ (z >> 31);
 }
 
-// float32 -> bf16 bits: nearest-even (seed == 0) or stochastic: 16 random bits
-// are added below the bf16 unit in the last place and the result truncated,
-// so the magnitude rounds up with probability equal to the dropped fraction.
-__device__ __forceinline__ uint16_t round_bf16(float x, uint64_t seed, uint64_t idx) {
+// float32 -> bf16 bits: nearest-even (seed == 0) or stochastic with the 16
+// random bits r: they are added below the bf16 unit in the last place and the
+// result truncated, so the magnitude rounds up with probability equal to the
+// dropped fraction.  Parameter i takes 16-bit lane (i mod 4) of the (i / 4)-th
+// SplitMix64 output (lane 0 = the least significant bits).
+__device__ __forceinline__ uint16_t round_bf16_bits(float x, bool sr, uint32_t r) {
   const uint32_t u = __float_as_uint(x);
-  if (seed == 0 || (u & 0x7f800000u) == 0x7f800000u) {
+  if (!sr || (u & 0x7f800000u) == 0x7f800000u) {
     unsigned short h;
     asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(x));
     return h;
   }
-  const uint32_t r = (uint32_t)(splitmix64_at(seed, idx) >> 48);
   return (uint16_t)((u + r) >> 16);
+}
+__device__ __forceinline__ uint16_t round_bf16(float x, uint64_t seed, uint64_t idx) {
+  const uint32_t r =
+      seed ? (uint32_t)(splitmix64_at(seed, idx >> 2) >> (16 * (idx & 3))) & 0xffffu : 0u;
+  return round_bf16_bits(x, seed != 0, r);
 }
 
 template <typename ThT>
@@ -192,10 +198,17 @@ __global__ void __launch_bounds__(NT) k3_ewma_bf16(bf16_t* __restrict__ tp,
       Elem<bf16_t>::unpack(ld_stream_v4(tp + 8 * i), x);
       load8<ThT>(th + 8 * i, y);
       uint16_t o[8];
+      const uint64_t g0 = idx0 + 8 * i;  // idx0 is a multiple of 8: two whole generator outputs
+      uint64_t r0 = 0, r1 = 0;
+      if (seed) {
+        r0 = splitmix64_at(seed, g0 >> 2);
+        r1 = splitmix64_at(seed, (g0 >> 2) + 1);
+      }
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         const float v = copy ? y[k] : fmaf(b, y[k] - x[k], x[k]);
-        o[k] = round_bf16(v, seed, idx0 + 8 * i + k);
+        const uint64_t r = k < 4 ? r0 : r1;
+        o[k] = round_bf16_bits(v, seed != 0, (uint32_t)(r >> (16 * (k & 3))) & 0xffffu);
       }
       st_stream_v4(tp + 8 * i, make_uint4(o[0] | ((uint32_t)o[1] << 16), o[2] | ((uint32_t)o[3] << 16),
                                           o[4] | ((uint32_t)o[5] << 16), o[6] | ((uint32_t)o[7] << 16)));
