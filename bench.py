@@ -123,10 +123,20 @@ class ClockSampler:
                 "samples": len(inside), "reasons": sorted(reasons)}
 
 
-def kernel_source_hash():
+KERNEL_SOURCES = {
+    "k1_token_logprob": ("occ_logprob.cu", "occ_common.cuh"),
+    "k2_decoupled_loss_fwd_bwd": ("occ_loss.cu", "occ_loss_common.cuh", "occ_common.cuh"),
+    "k12_decoupled_loss_fused": ("occ_fused.cu", "occ_loss_common.cuh", "occ_common.cuh"),
+    "k3_ewma_update": ("occ_ewma.cu", "occ_common.cuh"),
+}
+
+
+def kernel_source_hash(name):
+    """Hash of the sources a kernel is built from (its traffic capture stays
+    valid while they are unchanged)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2605_12070_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in KERNEL_SOURCES[name]:
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
@@ -134,15 +144,16 @@ def kernel_source_hash():
 
 def ncu_traffic():
     """Per-unit DRAM bytes from the committed ncu summary
-    (profiles/traffic_per_unit.json), if the kernels have not changed since it
-    was captured; {} otherwise."""
+    (profiles/traffic_per_unit.json) for the kernels whose sources have not
+    changed since the capture."""
     path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
     try:
         with open(path) as f:
             d = json.load(f)
     except Exception:
         return {}
-    return d.get("kernels", {}) if d.get("source_hash") == kernel_source_hash() else {}
+    return {k: v for k, v in d.get("kernels", {}).items()
+            if k in KERNEL_SOURCES and v.get("source_hash") == kernel_source_hash(k)}
 
 
 def traffic_bytes(tr, name, T, n_valid, n_params):

@@ -876,7 +876,7 @@ static int k2_threads() {
   return nt;
 }
 
-// Kernel variant for aligned rows: "l2" (default), "reg" or "tma"
+// Kernel variant for aligned rows: "l2" (default), "l2_1024", "reg" or "tma"
 // (OCC_K2_VARIANT overrides, for tuning).
 static int k2_variant() {
   static int v = [] {
@@ -925,8 +925,7 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     }();
     auto kern = (var == 3) ? k2_loss_l2<Tin, Tout, 1024, 8>
                            : (unroll == 4 ? k2_loss_l2<Tin, Tout, 512, 4>
-                                          : (unroll == 12 ? k2_loss_l2<Tin, Tout, 512, 12>
-                                                          : k2_loss_l2<Tin, Tout, 512, 8>));
+                                          : k2_loss_l2<Tin, Tout, 512, 8>);
     const int nt = (var == 3) ? 1024 : 512;
     if (head_bytes > 0) {
       cudaError_t e =

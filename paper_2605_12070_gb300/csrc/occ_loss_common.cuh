@@ -294,6 +294,100 @@ inline WsLayout ws_layout(int64_t T) {
 }
 
 
+// Online (c, s, sv): s = sum 2^(x L - c), sv = sum 2^(x L - c) v.
+struct LseAccV {
+  float c, s, sv;
+};
+
+template <int N, bool WV>
+__device__ __forceinline__ void accv_add(LseAccV& a, const float (&x)[N], const float (&v)[N]) {
+  float t = 0.f, tv = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    const float e = ex2_approx(fmaf(x[j], kLog2e, -a.c));
+    t += e;
+    if (WV) tv = fmaf(e, v[j], tv);
+  }
+  if (t <= 1.8446744073709552e19f) {  // 2^64; false for inf / NaN and for c = -inf
+    a.s += t;
+    a.sv += tv;
+    return;
+  }
+  float m = x[0];
+#pragma unroll
+  for (int j = 1; j < N; ++j) m = fmaxf(m, x[j]);
+  const float ms = m * kLog2e;
+  if (ms > a.c + kRescale) {
+    const float f = exp2f(a.c - ms);
+    a.s *= f;
+    a.sv *= f;
+    a.c = ms;
+  }
+  if (a.c == -INFINITY) return;
+  t = 0.f;
+  tv = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    const float e = ex2_approx(fmaf(x[j], kLog2e, -a.c));
+    t += e;
+    if (WV) tv = fmaf(e, v[j], tv);
+  }
+  a.s += t;
+  a.sv += tv;
+}
+
+struct FusedRed {
+  float c[2][32];
+  float2 s[2][32];
+  float sv[2][32];
+};
+
+// Block merge of two accumulators; the results are valid in thread 0.
+template <int NT>
+__device__ __forceinline__ void block_lse_v2(const LseAccV (&acc)[2], FusedRed& r, float (&C)[2],
+                                             float2 (&S)[2], float (&SV)[2]) {
+  constexpr int NW = NT / 32;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const float wm = warp_max(acc[k].c);
+    const float f = acc[k].c == -INFINITY ? 0.f : exp2f(acc[k].c - wm);
+    float2 v = warp_pair_sum(make_float2(acc[k].s * f, 0.f));
+    float sv = acc[k].sv * f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, o);
+    if (lane == 0) {
+      r.c[k][wid] = wm;
+      r.s[k][wid] = v;
+      r.sv[k][wid] = sv;
+    }
+  }
+  __syncthreads();
+  if (wid == 0) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const float cw = lane < NW ? r.c[k][lane] : -INFINITY;
+      const float cm = warp_max(cw);
+      float2 w = make_float2(0.f, 0.f);
+      float sv = 0.f;
+      if (lane < NW && cw != -INFINITY) {
+        const float f = exp2f(cw - cm);
+        const float2 p = r.s[k][lane];
+        const float hi = p.x * f;
+        w = make_float2(hi, fmaf(p.x, f, -hi) + p.y * f);
+        sv = r.sv[k][lane] * f;
+      }
+      w = warp_pair_sum(w);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, o);
+      C[k] = cm;
+      S[k] = w;
+      SV[k] = sv;
+    }
+  }
+}
+
+
 // Host: validates the arguments every loss entry point shares (all but the
 // source of log pi_old), fills the kernel arguments and reports whether the
 // rows qualify for the 16-byte vector kernels.
