@@ -48,6 +48,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--tau", type=float, default=0.5)
     ap.add_argument("--tokens", type=int, default=None, help="resize T (profiling runs only)")
+    ap.add_argument("--ewma-variants", action="store_true",
+                    help="instead of the step, time the bf16 and host-resident EWMA buffers")
     ap.add_argument("--loss-path", default="fused", choices=["fused", "two-call"],
                     help="fused: one launch reads old and current logits (occ_decoupled_loss_fused); "
                          "two-call: occ_token_logprob then occ_decoupled_loss_fwd_bwd")
@@ -285,6 +287,10 @@ def main():
     if args.impl == "reference":
         run_reference(args, batch, world)
         return
+    if args.ewma_variants:
+        del batch
+        run_ewma_variants(args, dev)
+        return
 
     theta, theta_prox = make_ewma_buffers(args.ewma_n, seed=rank, device=dev)
     state = occ.new_ewma_state(dev, w0=1.0 / (1.0 - EWMA_BETA))
@@ -513,6 +519,59 @@ def run_e2e(args, batch, theta, theta_prox, state, stats, loss_fn, world, dev):
     return {"value": round(world * batch.T / sec, 1), "unit": "tokens/s",
             "h2d_bytes_per_step": need, "d2h_bytes_per_step": occ.LOSS_STATS_BYTES,
             "ms_per_step": round(sec * 1e3, 3), "steps": args.e2e_steps}
+
+
+def run_ewma_variants(args, dev):
+    """Times the bf16 proximal buffer (nearest and stochastic rounding, fp32 and
+    bf16 theta) on --ewma-n parameters and the pinned-host buffer on 2e9."""
+    import torch
+
+    from paper_2605_12070_gb300 import occ
+    from paper_2605_12070_gb300.workloads import make_ewma_buffers
+
+    def timeit(fn, reps=5, warm=2):
+        for _ in range(warm):
+            fn()
+        torch.cuda.synchronize()
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(reps):
+            fn()
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) / reps
+
+    peak, peak_kind = measured_peak()
+    n = args.ewma_n
+    th, tp = make_ewma_buffers(n, seed=0, device=dev)
+    tpb = tp.to(torch.bfloat16)
+    del tp
+    st = occ.new_ewma_state(dev, w0=1.0 / (1.0 - EWMA_BETA))
+    out = {"metric": "PPO-EWMA update variants", "unit": "ms", "n_params": n,
+           "peak_gbs": peak, "peak_kind": peak_kind}
+    for name, fn, bpp in (
+            ("bf16_buffer_f32_theta_nearest",
+             lambda: occ.occ_ewma_update_bf16(tpb, th, EWMA_BETA, st, sr_seed=0), 8),
+            ("bf16_buffer_f32_theta_stochastic",
+             lambda: occ.occ_ewma_update_bf16(tpb, th, EWMA_BETA, st, sr_seed=77), 8)):
+        ms = timeit(fn)
+        out[name] = {"ms": round(ms, 3), "frac": round(n * bpp / ms / 1e6 / peak, 4)}
+    thb = th.to(torch.bfloat16)
+    del th
+    ms = timeit(lambda: occ.occ_ewma_update_bf16(tpb, thb, EWMA_BETA, st, sr_seed=77))
+    out["bf16_buffer_bf16_theta_stochastic"] = {"ms": round(ms, 3),
+                                                "frac": round(n * 6 / ms / 1e6 / peak, 4)}
+    del tpb
+    m = min(n, 2_000_000_000)
+    host = torch.empty(m, dtype=torch.bfloat16, pin_memory=True)
+    host.copy_(thb[:m])
+    staging = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    s1 = torch.cuda.Stream(dev)
+    ms = timeit(lambda: occ.occ_ewma_update_host(host, thb[:m], EWMA_BETA, st, staging, sr_seed=5,
+                                                 stream1=s1), reps=3, warm=1)
+    out["host_bf16_buffer"] = {"ms": round(ms, 3), "n_params": m, "staging_bytes": 256 << 20,
+                               "host_device_gbs": round(2 * m * 2 / ms / 1e6, 1)}
+    print(json.dumps(out), flush=True)
 
 
 def run_reference(args, batch, world):
