@@ -91,6 +91,9 @@ def test_streak_rule():
     assert resets == [(False, 1), (False, 0), (False, 1), (True, 0), (False, 0), (False, 1)]
     _, _, reset, _ = ewma_coefficients(EwmaState(w=2.0), 0.75, force_reset=True)
     assert reset
+    # Sec. 5.2 resets when rho < tau: rho exactly at tau does not count as low
+    _, _, reset, st = ewma_coefficients(EwmaState(w=2.0), 0.75, n_active=9, n_valid=10, tau=0.9)
+    assert 9 / 10 == 0.9 and not reset and st.streak == 0
 
 
 # ---------------------------------------------------------------- bf16 buffers

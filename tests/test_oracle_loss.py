@@ -308,3 +308,30 @@ def test_proxy_ratio_closed_forms():
     for kind in ("loglinear", "arithmetic"):
         np.testing.assert_allclose(proxy_logprob(kind, 0.0, lmu, lth), lth, atol=1e-13)
         np.testing.assert_allclose(proxy_logprob(kind, 1.0, lmu, lth), lmu, atol=1e-13)
+
+
+def test_thresholds_inclusive_at_the_exact_bound():
+    """Eq. 4's M_[1/c,c] and Eq. 3's r_s <= 1 + eps (A >= 0) / r_s >= 1 - eps (A < 0)
+    include the bound itself.  The bounds are chosen as exp(d) of the very
+    log-ratio d the oracle will see, so the ratio equals the bound exactly."""
+    lmu = np.array([-2.0, -2.0])
+    d = np.array([0.125, -0.25])             # log r_d at the upper / lower band edge
+    lold = lmu + d
+    assert np.all(lold - lmu == d)
+    p = LossParams(rd_lo=float(np.exp(d[1])), rd_hi=float(np.exp(d[0])), eps_low=0.2,
+                   eps_high=0.28)
+    out = token_terms(lold, lold, lmu, np.array([1.0, 1.0]), None, p)
+    assert out["r_d"][0] == p.rd_hi and out["r_d"][1] == p.rd_lo
+    assert np.all(out["in_band"])
+    # clip bounds hit exactly: r_s = exp(ds) in [1, 2) so that 1 + (exp(ds) - 1) == exp(ds)
+    ds, dl = 0.25, -0.125
+    up = float(np.exp(ds))
+    lo = float(np.exp(dl))
+    lth = np.array([-3.0 + ds, -3.0 + dl])
+    lold = np.array([-3.0, -3.0])
+    assert np.all(lth - lold == np.array([ds, dl]))
+    p = LossParams(rd_lo=0.5, rd_hi=2.0, eps_low=1.0 - lo, eps_high=up - 1.0)
+    assert 1.0 + p.eps_high == up and 1.0 - p.eps_low == lo
+    out = token_terms(lth, lold, lold, np.array([1.0, -1.0]), None, p)
+    assert out["r_s"][0] == up and out["r_s"][1] == lo
+    assert np.all(out["mis"]) and out["n_clipped"] == 0
