@@ -65,7 +65,6 @@ __device__ __forceinline__ void backward_slice(const uint4* sv, int64_t nvec, in
   }
 }
 
-constexpr uint64_t kCopyTimeoutNs = 2000000000ull;  // a row slice lands in microseconds
 
 // Persistent, TMA-pipelined cluster kernel.  Cluster c of the grid handles rows
 // c, c + ncl, c + 2 ncl, ...; CTA `rank` of the cluster owns columns
@@ -125,7 +124,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_tma(const K2Args a) {
   if (tid == 0 && bulk > 0)
     for (int st = 0; st < STAGES - 1; ++st) {
       const int64_t r = cid + (int64_t)st * ncl;
-      if (r < T && row_ok(r)) issue(r, st);
+      if (r < T && r != a.lost_copy_row && row_ok(r)) issue(r, st);
     }
 
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
@@ -137,7 +136,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_tma(const K2Args a) {
     if (tid == 0 && bulk > 0 && !fault) {
       const int64_t r = row + (int64_t)(STAGES - 1) * ncl;
       const int sn = (k + STAGES - 1) % STAGES;
-      if (r < T && row_ok(r)) issue(r, sn);
+      if (r < T && r != a.lost_copy_row && row_ok(r)) issue(r, sn);
     }
     const int id = a.ids[row];
     const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
@@ -157,7 +156,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_tma(const K2Args a) {
     unsigned char* sp = smem_raw + (size_t)st * stage_bytes;
     if (bulk > 0) {
       const uint32_t par = (phase >> st) & 1u;
-      const bool ok = mbar_wait_bounded(&bars[st], par, fault ? 0 : kCopyTimeoutNs);
+      const bool ok = mbar_wait_bounded(&bars[st], par, fault ? 0 : a.wait_ns);
       phase ^= 1u << st;
       if (!ok) fault = true;
       if (tid == 0 && ok) pend &= ~(1u << st);
@@ -277,7 +276,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_tma(const K2Args a) {
     // copies still in flight (only after a timeout): wait, bounded, before exiting
     for (int st = 0; st < STAGES; ++st)
       if (pend & (1u << st)) {
-        if (!mbar_wait_bounded(&bars[st], (ppar >> st) & 1u, kCopyTimeoutNs))
+        if (!mbar_wait_bounded(&bars[st], (ppar >> st) & 1u, a.wait_ns))
           atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
       }
   }
@@ -365,13 +364,13 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
   auto refill = [&](int64_t row, int st) {
     if (tid == 0 && bulk > 0 && !fault) {
       const int64_t r = row + (int64_t)STAGES * ncl;
-      if (r < T && row_ok(r)) issue(r, st);
+      if (r < T && r != a.lost_copy_row && row_ok(r)) issue(r, st);
     }
   };
   if (tid == 0 && bulk > 0)
     for (int st = 0; st < STAGES; ++st) {
       const int64_t r = cid + (int64_t)st * ncl;
-      if (r < T && row_ok(r)) issue(r, st);
+      if (r < T && r != a.lost_copy_row && row_ok(r)) issue(r, st);
     }
 
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
@@ -398,7 +397,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
     }
     const unsigned char* sp = smem_raw + (size_t)st * stage_bytes;
     if (bulk > 0) {
-      const bool ok = mbar_wait_bounded(&bars[st], (phase >> st) & 1u, fault ? 0 : kCopyTimeoutNs);
+      const bool ok = mbar_wait_bounded(&bars[st], (phase >> st) & 1u, fault ? 0 : a.wait_ns);
       phase ^= 1u << st;
       if (!ok) fault = true;
       if (tid == 0 && ok) pend &= ~(1u << st);
@@ -547,7 +546,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
     if (fault) atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
     for (int st = 0; st < STAGES; ++st)
       if (pend & (1u << st)) {
-        if (!mbar_wait_bounded(&bars[st], (ppar >> st) & 1u, kCopyTimeoutNs))
+        if (!mbar_wait_bounded(&bars[st], (ppar >> st) & 1u, a.wait_ns))
           atomicOr(a.ws_err, OCC_DATA_ERR_TIMEOUT);
       }
   }
@@ -820,6 +819,11 @@ static int max_active_clusters(const void* kern, int C, int NT, size_t smem) {
 template <typename Kern>
 static occ_status launch_persistent(Kern kern, int NT, K2Args a, const ClusterPlan& pl, int stages,
                                     cudaStream_t s) {
+  // Test hooks of the bounded waits: OCC_TEST_LOST_COPY_ROW makes the producer
+  // skip one row's copy so that its consumers' wait runs out (after
+  // OCC_TEST_WAIT_TIMEOUT_NS); the kernel then reports OCC_DATA_ERR_TIMEOUT.
+  if (const char* e = getenv("OCC_TEST_LOST_COPY_ROW")) a.lost_copy_row = atoll(e);
+  if (const char* e = getenv("OCC_TEST_WAIT_TIMEOUT_NS")) a.wait_ns = strtoull(e, nullptr, 10);
   const size_t smem = (size_t)stages * pl.stage_bytes;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess)

@@ -43,6 +43,8 @@ struct K2Args {
   int64_t T, V, ld, S, row0;
   int64_t stage_bytes;  // shared-memory bytes of one pipeline stage (TMA kernel)
   int* ws_err;          // device-detected error bits, OR-ed into stats.err
+  uint64_t wait_ns;     // limit of each wait for an asynchronous copy (cluster kernels)
+  int64_t lost_copy_row;  // test hook (-1 = off): the copy of this row is never issued
   const int32_t* ids;
   const float* lp_old;
   const float* lp_mu;
@@ -447,6 +449,8 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   a.S = V;
   a.row0 = 0;
   a.stage_bytes = 0;
+  a.wait_ns = 2000000000ull;
+  a.lost_copy_row = -1;
   a.ids = ids;
   a.lp_old = nullptr;
   a.lp_mu = logp_mu;
