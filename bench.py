@@ -43,6 +43,8 @@ def parse_args():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--ewma-n", type=int, default=7_600_000_000)
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-graph", action="store_true",
+                    help="skip timing the step replayed from a captured CUDA graph")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -384,6 +386,25 @@ def main():
     alt_k1 = sum(e[0].elapsed_time(e[1]) for e in aevs) / 10 / 1e3
     alt_k2 = sum(e[1].elapsed_time(e[2]) for e in aevs) / 10 / 1e3
 
+    # the same step captured once as a CUDA graph and replayed (no host work per step)
+    graph = None
+    if world == 1 and not args.no_graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            step()
+        for _ in range(2):
+            g.replay()
+        gs, ge = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        gs.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        ge.record(stream)
+        torch.cuda.synchronize()
+        gsec = gs.elapsed_time(ge) / 1e3 / args.steps
+        graph = {"ms_per_step": round(gsec * 1e3, 4), "tokens_per_s": round(T / gsec, 1),
+                 "steps": args.steps,
+                 "launches_per_replay": 5 if args.loss_path == "fused" else 6}
+
     peak, peak_kind = measured_peak()
     traffic = ncu_traffic()
     bytes_k1 = T * V * 2 + T * 8
@@ -450,6 +471,7 @@ def main():
                       "hbm_frac": round(loss_bytes / (k1 + k2) / 1e9 / peak, 4)},
         "loss_only_other_path": alt,
         "gpu_launches": args.steps * (5 if args.loss_path == "fused" else 6),
+        "graph_replay": graph,
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
