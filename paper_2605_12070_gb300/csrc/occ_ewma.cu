@@ -159,32 +159,48 @@ __device__ __forceinline__ uint16_t round_bf16(float x, uint64_t seed, uint64_t 
   return round_bf16_bits(x, seed != 0, r);
 }
 
+// Eight theta values as loaded (raw 16-byte words) and unpacked to float.
 template <typename ThT>
-__device__ __forceinline__ void load8(const ThT* p, float (&x)[8]);
+struct Raw8;
 template <>
-__device__ __forceinline__ void load8<float>(const float* p, float (&x)[8]) {
-  const uint4 a = ld_stream_v4(p), b = ld_stream_v4(p + 4);
-  x[0] = __uint_as_float(a.x); x[1] = __uint_as_float(a.y);
-  x[2] = __uint_as_float(a.z); x[3] = __uint_as_float(a.w);
-  x[4] = __uint_as_float(b.x); x[5] = __uint_as_float(b.y);
-  x[6] = __uint_as_float(b.z); x[7] = __uint_as_float(b.w);
-}
+struct Raw8<float> {
+  uint4 a, b;
+  __device__ __forceinline__ void load(const float* p) {
+    a = ld_stream_v4(p);
+    b = ld_stream_v4(p + 4);
+  }
+  __device__ __forceinline__ void unpack(float (&x)[8]) const {
+    x[0] = __uint_as_float(a.x); x[1] = __uint_as_float(a.y);
+    x[2] = __uint_as_float(a.z); x[3] = __uint_as_float(a.w);
+    x[4] = __uint_as_float(b.x); x[5] = __uint_as_float(b.y);
+    x[6] = __uint_as_float(b.z); x[7] = __uint_as_float(b.w);
+  }
+};
 template <>
-__device__ __forceinline__ void load8<bf16_t>(const bf16_t* p, float (&x)[8]) {
-  Elem<bf16_t>::unpack(ld_stream_v4(p), x);
-}
+struct Raw8<bf16_t> {
+  uint4 a;
+  __device__ __forceinline__ void load(const bf16_t* p) { a = ld_stream_v4(p); }
+  __device__ __forceinline__ void unpack(float (&x)[8]) const { Elem<bf16_t>::unpack(a, x); }
+};
 __device__ __forceinline__ float load1(const float* p) { return *p; }
 __device__ __forceinline__ float load1(const bf16_t* p) {
   return __uint_as_float(((uint32_t)p->bits) << 16);
 }
 
 // theta_prox (bf16, 16-byte aligned) <- theta_prox + b (theta - theta_prox),
-// eight parameters per thread iteration; elements [8 n8, n) in a scalar tail.
-template <typename ThT, int NT>
-__global__ void __launch_bounds__(NT) k3_ewma_bf16(bf16_t* __restrict__ tp,
-                                                   const ThT* __restrict__ th, int64_t n,
-                                                   bool vec, const occ_ewma_state* __restrict__ st,
-                                                   uint64_t seed, uint64_t idx0) {
+// eight parameters per vector, U vectors of each operand in flight per thread;
+// elements [8 n8, n) in a scalar tail.  On a copy step (b = 1) theta_prox is
+// not read.
+// Resident CTAs per SM: the launcher sizes the grid to one full wave of them.
+template <typename ThT>
+constexpr int k3_bf16_ctas_per_sm() {
+  return sizeof(ThT) == 4 ? 3 : 4;
+}
+
+template <typename ThT, int NT, int U>
+__global__ void __launch_bounds__(NT, k3_bf16_ctas_per_sm<ThT>())
+    k3_ewma_bf16(bf16_t* __restrict__ tp, const ThT* __restrict__ th, int64_t n, bool vec,
+                 const occ_ewma_state* __restrict__ st, uint64_t seed, uint64_t idx0) {
   const double bd = st->coef_b;
   const bool copy = (bd == 1.0);
   const float b = (float)bd;
@@ -193,12 +209,12 @@ __global__ void __launch_bounds__(NT) k3_ewma_bf16(bf16_t* __restrict__ tp,
   int64_t done = 0;
   if (vec) {
     const int64_t n8 = n / 8;
-    for (int64_t i = gtid; i < n8; i += stride) {
+    auto emit = [&](int64_t iv, const uint4& xr, const Raw8<ThT>& yr) {
       float x[8], y[8];
-      Elem<bf16_t>::unpack(ld_stream_v4(tp + 8 * i), x);
-      load8<ThT>(th + 8 * i, y);
+      Elem<bf16_t>::unpack(xr, x);
+      yr.unpack(y);
       uint16_t o[8];
-      const uint64_t g0 = idx0 + 8 * i;  // idx0 is a multiple of 8: two whole generator outputs
+      const uint64_t g0 = idx0 + 8 * iv;  // idx0 is a multiple of 8: two whole generator outputs
       uint64_t r0 = 0, r1 = 0;
       if (seed) {
         r0 = splitmix64_at(seed, g0 >> 2);
@@ -210,14 +226,31 @@ __global__ void __launch_bounds__(NT) k3_ewma_bf16(bf16_t* __restrict__ tp,
         const uint64_t r = k < 4 ? r0 : r1;
         o[k] = round_bf16_bits(v, seed != 0, (uint32_t)(r >> (16 * (k & 3))) & 0xffffu);
       }
-      st_stream_v4(tp + 8 * i, make_uint4(o[0] | ((uint32_t)o[1] << 16), o[2] | ((uint32_t)o[3] << 16),
-                                          o[4] | ((uint32_t)o[5] << 16), o[6] | ((uint32_t)o[7] << 16)));
+      st_stream_v4(tp + 8 * iv, make_uint4(o[0] | ((uint32_t)o[1] << 16), o[2] | ((uint32_t)o[3] << 16),
+                                           o[4] | ((uint32_t)o[5] << 16), o[6] | ((uint32_t)o[7] << 16)));
+    };
+    int64_t i = gtid;
+    for (; i + (int64_t)(U - 1) * stride < n8; i += (int64_t)U * stride) {
+      uint4 xr[U];
+      Raw8<ThT> yr[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        yr[u].load(th + 8 * (i + u * stride));
+        xr[u] = copy ? make_uint4(0, 0, 0, 0) : ld_stream_v4(tp + 8 * (i + u * stride));
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) emit(i + u * stride, xr[u], yr[u]);
+    }
+    for (; i < n8; i += stride) {
+      Raw8<ThT> yr;
+      yr.load(th + 8 * i);
+      emit(i, copy ? make_uint4(0, 0, 0, 0) : ld_stream_v4(tp + 8 * i), yr);
     }
     done = n8 * 8;
   }
   for (int64_t i = done + gtid; i < n; i += stride) {
-    const float x = load1(tp + i), y = load1(th + i);
-    const float v = copy ? y : fmaf(b, y - x, x);
+    const float y = load1(th + i);
+    const float v = copy ? y : fmaf(b, y - load1(tp + i), load1(tp + i));
     tp[i].bits = round_bf16(v, seed, idx0 + i);
   }
 }
@@ -298,14 +331,18 @@ occ_status launch_bf16_body(bf16_t* tp, const void* th, occ_dtype theta_dt, int6
   if (n == 0) return OCC_OK;
   const bool vec = aligned(tp, 16) && aligned(th, 16);
   const int64_t work = vec ? (n + 7) / 8 : n;
-  const int64_t need = (work + kK3Threads - 1) / kK3Threads;
-  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, (int64_t)sm_count() * 8));
+  const int64_t need = (work + kK3Threads * kK3Unroll - 1) / (kK3Threads * kK3Unroll);
+  auto grid_for = [&](int per_sm) {
+    return (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, (int64_t)sm_count() * per_sm));
+  };
   if (theta_dt == OCC_BF16)
-    k3_ewma_bf16<bf16_t, kK3Threads><<<grid, kK3Threads, 0, s>>>(tp, (const bf16_t*)th, n, vec, st,
-                                                                 seed, idx0);
+    k3_ewma_bf16<bf16_t, kK3Threads, kK3Unroll>
+        <<<grid_for(k3_bf16_ctas_per_sm<bf16_t>()), kK3Threads, 0, s>>>(tp, (const bf16_t*)th, n,
+                                                                         vec, st, seed, idx0);
   else
-    k3_ewma_bf16<float, kK3Threads><<<grid, kK3Threads, 0, s>>>(tp, (const float*)th, n, vec, st,
-                                                                seed, idx0);
+    k3_ewma_bf16<float, kK3Threads, kK3Unroll>
+        <<<grid_for(k3_bf16_ctas_per_sm<float>()), kK3Threads, 0, s>>>(tp, (const float*)th, n,
+                                                                        vec, st, seed, idx0);
   return check_launch("k3_ewma_bf16");
 }
 
