@@ -175,11 +175,11 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
         for (; k + (int64_t)(2 * U - 1) * NT < nre; k += (int64_t)2 * U * NT) {
           uint4 r[2 * U];
 #pragma unroll
-          for (int u = 0; u < 2 * U; ++u) r[u] = ld_hint_v4(zv + (nvec - 1 - (k + u * NT)), last);
+          for (int u = 0; u < 2 * U; ++u) r[u] = ld_hint_v4(zv + (head + (k + u * NT)), last);
 #pragma unroll
-          for (int u = 0; u < 2 * U; ++u) emit(nvec - 1 - (k + u * NT), r[u]);
+          for (int u = 0; u < 2 * U; ++u) emit(head + (k + u * NT), r[u]);
         }
-        for (; k < nre; k += NT) emit(nvec - 1 - k, ld_hint_v4(zv + (nvec - 1 - k), last));
+        for (; k < nre; k += NT) emit(head + k, ld_hint_v4(zv + (head + k), last));
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
         if ((int64_t)tid < V - tail0) {

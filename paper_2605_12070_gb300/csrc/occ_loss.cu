@@ -556,9 +556,11 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
 // row kept in shared memory.  The forward pass reads the row from HBM once:
 // its first `head` vectors are also stored in shared memory, the rest is read
 // with an L2 evict-last policy.  The backward pass takes the head from shared
-// memory and re-reads only the remainder, newest data first and with an
+// memory and re-reads only the remainder, oldest data first and with an
 // evict-first policy (its last use), so the re-read is served by L2 and HBM
-// sees the logits once and dlogits once.  dlogits are written evict-first.
+// sees the logits once and dlogits once.  Oldest-first bounds the time a line
+// waits in L2 by the longer of the two passes (newest-first lets the first
+// lines wait through both).  dlogits are written evict-first.
 template <typename Tin, typename Tout, int NT, int U>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   constexpr int VEC = Elem<Tin>::kVec;
@@ -665,17 +667,17 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
           }
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
-        // re-read part, newest first: vectors nvec-1-tid, nvec-1-tid-NT, ... >= head
+        // re-read part, oldest first: vectors head+tid, head+tid+NT, ... < nvec
         const int64_t nre = nvec - head;
         int64_t k = tid;
         for (; k + (int64_t)(U - 1) * NT < nre; k += (int64_t)U * NT) {
           uint4 r[U];
 #pragma unroll
-          for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + (nvec - 1 - (k + u * NT)), last);
+          for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + (head + (k + u * NT)), last);
 #pragma unroll
-          for (int u = 0; u < U; ++u) emit(nvec - 1 - (k + u * NT), r[u]);
+          for (int u = 0; u < U; ++u) emit(head + (k + u * NT), r[u]);
         }
-        for (; k < nre; k += NT) emit(nvec - 1 - k, ld_hint_v4(zv + (nvec - 1 - k), last));
+        for (; k < nre; k += NT) emit(head + k, ld_hint_v4(zv + (head + k), last));
         // on-chip head
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);

@@ -111,3 +111,30 @@ def test_proxy_rejected_by_fused_entry_point():
         ctypes.c_void_p(b.adv.data_ptr()), None, ctypes.byref(p), None, None, None, None, None,
         None, 0, ctypes.c_void_p(st.data_ptr()), ctypes.c_void_p(ws.data_ptr()), ws.numel(), None)
     assert rc == 1 and b"proxies" in lib.occ_last_error()
+
+
+@pytest.mark.parametrize("kind", ["loglinear", "arithmetic"])
+@pytest.mark.parametrize("alpha", [0.0, 1.0])
+def test_proxy_degenerate_weights(kind, alpha):
+    # alpha = 1: the proxy is mu_old itself, so r_d = 1 and no token leaves the
+    # band (Eq. 4 reduces to plain PPO-clip).  alpha = 0: the proxy is pi_theta,
+    # so r_s = 1 and no token is clipped (Table 1's interpolation end points).
+    b = make_loss_batch("agentic_bf16_v151936", T=256, seed=13, device="cuda")
+    rows = np.arange(b.T)
+    lt64, lse = logprob_rows(b.z_theta, b.ids, rows)
+    lmu = b.logp_mu.cpu().numpy().astype(np.float64)
+    lp_prox = orc.proxy_logprob(kind, alpha, lmu, np.nan_to_num(lt64))
+    o = oracle_loss(b, lt64, lp_prox, loss_params(b))
+    out = occ.occ_decoupled_loss_fwd_bwd(b.z_theta, b.ids, None, b.logp_mu, b.adv, b.mask,
+                                         proxy=kind, alpha=alpha, **b.thresholds())
+    torch.cuda.synchronize()
+    st = occ.decode_loss_stats(out["stats"])
+    fl = out["flags"].cpu().numpy()
+    assert st.n_valid == o["n_valid"] > 0
+    if alpha == 1.0:
+        assert st.n_rd_out == 0 == o["n_rd_out"]
+    else:
+        assert st.n_clipped == 0 == o["n_clipped"]
+    near = np.minimum(o["dist_rd"], o["dist_rs"]) <= 1e-6
+    assert not ((fl != o["flags"]) & ~(near & o["valid"])).any()
+    assert abs(st.loss - o["loss"]) <= 1e-4 * abs(o["loss"]) + 1e-12
