@@ -306,6 +306,29 @@ occ_status occ_ewma_update_host(void* theta_prox_host, occ_dtype prox_dt, const 
  * empty history, 1/(1-beta) to start in the stationary regime. */
 occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* stream);
 
+/*
+ * occ_host_alloc / occ_host_free -- a PINNED HOST buffer for the inputs of an
+ * end-to-end step.  This is host plumbing: the paper has no counterpart.
+ *
+ * occ_host_alloc maps `bytes` (rounded up to the host's transparent-huge-page
+ * size) of anonymous memory starting on a huge-page boundary, advises the
+ * kernel to back it with huge pages and page-locks it with cudaHostRegister.
+ * The buffer is an ordinary page-locked buffer for cudaMemcpyAsync and for
+ * occ_ewma_update_host; huge pages only cut the host link's address
+ * translation when copies stream through tens of GB.  If the kernel declines
+ * huge pages the buffer is backed by base pages and works the same, slower.
+ * Contents are zero.  *out receives the pointer, or NULL on failure.
+ * Returns OCC_ERR_INVALID_ARG for bytes == 0 or a failed mmap and
+ * OCC_ERR_CUDA if the memory cannot be registered (no device, or no
+ * page-lockable memory left); nothing stays mapped after a failure.
+ *
+ * occ_host_free unregisters and unmaps a buffer from occ_host_alloc; `bytes`
+ * is the size passed to occ_host_alloc.  The caller must make sure no copy
+ * from or to it is still in flight.  NULL is a no-op.
+ */
+occ_status occ_host_alloc(size_t bytes, void** out);
+occ_status occ_host_free(void* ptr, size_t bytes);
+
 /* Static description of a status code. */
 const char* occ_status_string(occ_status s);
 

@@ -11,8 +11,10 @@ CUDA device, the call raises.
 """
 
 import ctypes
+import math
 import os
 import struct
+import weakref
 from dataclasses import dataclass
 
 import torch
@@ -34,7 +36,8 @@ _STATE_FMT = "<3d4i"
 EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_fwd_bwd",
            "occ_decoupled_loss_fused", "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update",
            "occ_ewma_update_bf16", "occ_ewma_update_host", "occ_ewma_state_init",
-           "occ_status_string", "occ_last_error", "occ_version")
+           "occ_host_alloc", "occ_host_free", "occ_status_string", "occ_last_error",
+           "occ_version")
 
 
 class OccError(RuntimeError):
@@ -101,6 +104,10 @@ def lib():
     L.occ_ewma_update_host.restype = i32
     L.occ_ewma_state_init.argtypes = [vp, dbl, vp]
     L.occ_ewma_state_init.restype = i32
+    L.occ_host_alloc.argtypes = [ctypes.c_size_t, ctypes.POINTER(vp)]
+    L.occ_host_alloc.restype = i32
+    L.occ_host_free.argtypes = [vp, ctypes.c_size_t]
+    L.occ_host_free.restype = i32
     L.occ_status_string.argtypes = [i32]
     L.occ_status_string.restype = ctypes.c_char_p
     L.occ_last_error.argtypes = []
@@ -407,3 +414,28 @@ def occ_ewma_update_host(theta_prox_host, theta, beta, state, staging, stats=Non
         ctypes.c_void_p(s0.cuda_stream), ctypes.c_void_p(s1.cuda_stream))
     _check(rc, "occ_ewma_update_host")
     return theta_prox_host
+
+
+def _host_free(ptr, nbytes):
+    lib().occ_host_free(ctypes.c_void_p(ptr), nbytes)
+
+
+def occ_host_alloc(shape, dtype):
+    """Pinned host tensor from occ_host_alloc (huge-page backed, zero-filled).
+
+    The memory is released through occ_host_free when the last tensor or view
+    of it is gone; copies from or to it must have completed by then."""
+    if isinstance(shape, int):
+        shape = (shape,)
+    elem = torch.empty((), dtype=dtype).element_size()
+    nbytes = math.prod(shape) * elem
+    if nbytes == 0:
+        return torch.empty(shape, dtype=dtype, pin_memory=True)
+    # torch reports a registered range as pinned (and copies it asynchronously)
+    # only once its own CUDA state exists
+    torch.cuda.init()
+    ptr = ctypes.c_void_p()
+    _check(lib().occ_host_alloc(nbytes, ctypes.byref(ptr)), "occ_host_alloc")
+    buf = (ctypes.c_uint8 * nbytes).from_address(ptr.value)
+    weakref.finalize(buf, _host_free, ptr.value, nbytes)
+    return torch.frombuffer(buf, dtype=torch.uint8).view(dtype).view(shape)

@@ -83,3 +83,21 @@ def test_no_cpu_fallback():
     import torch
     with pytest.raises(occ.OccError, match="CUDA"):
         occ.occ_token_logprob(torch.zeros(2, 4), torch.zeros(2, dtype=torch.int32))
+
+
+def test_host_alloc_argument_checks(L):
+    p = ctypes.c_void_p(1)
+    assert L.occ_host_alloc(0, ctypes.byref(p)) == 1 and p.value is None
+    assert b"bytes == 0" in L.occ_last_error()
+    assert L.occ_host_alloc(1 << 20, None) == 1
+    assert L.occ_host_free(None, 0) == 0
+    assert L.occ_host_free(ctypes.c_void_p(4096 + 1), 1 << 20) == 1  # not from occ_host_alloc
+
+
+def test_host_alloc_fails_cleanly_without_a_device(L):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a device is present")
+    p = ctypes.c_void_p()
+    assert L.occ_host_alloc(1 << 20, ctypes.byref(p)) == 4  # OCC_ERR_CUDA
+    assert p.value is None and b"cudaHostRegister" in L.occ_last_error()
