@@ -15,7 +15,8 @@
  *
  * Conventions shared by every entry point:
  *   - Every pointer argument is caller-owned DEVICE memory unless marked
- *     "host".  The library never allocates or frees memory.
+ *     "host".  No entry point of the path allocates or frees memory (the
+ *     host-buffer helpers occ_host_alloc / occ_host_free exist for that).
  *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
  *     default stream).  A returned OCC_OK means the work was enqueued.
  *   - Arguments are validated on the host before anything is launched; an
