@@ -153,9 +153,13 @@ def token_terms(logp_theta, logp_old, logp_mu, adv, mask, params, id_ok=None, N=
              + active * FLAG_ACTIVE + FLAG_VALID).astype(np.uint8)
     flags = np.where(valid, flags, 0).astype(np.uint8)
 
-    dist_rd = np.minimum(np.abs(log_rd - np.log(p.rd_lo)), np.abs(log_rd - np.log(p.rd_hi)))
-    dist_rs = np.where(A >= 0, np.abs(log_rs - np.log1p(p.eps_high)),
-                       np.abs(log_rs - np.log1p(-p.eps_low)))
+    # distance (in log space) to the nearer band edge; an open edge (rd_lo = 0 or
+    # rd_hi = inf: Table 5's unmasked r_2 roles) is infinitely far
+    log_lo = np.log(p.rd_lo) if p.rd_lo > 0 else -np.inf
+    log_hi = np.log(p.rd_hi) if np.isfinite(p.rd_hi) else np.inf
+    dist_rd = np.minimum(np.abs(log_rd - log_lo), np.abs(log_rd - log_hi))
+    log_clip_lo = np.log1p(-p.eps_low) if p.eps_low < 1.0 else -np.inf  # eps_low = 1: no lower edge
+    dist_rs = np.where(A >= 0, np.abs(log_rs - np.log1p(p.eps_high)), np.abs(log_rs - log_clip_lo))
     return dict(
         log_rd=log_rd, log_rs=log_rs, r_d=r_d, r_s=r_s, in_band=in_band, mis=mis,
         valid=valid, loss_t=loss_t, g=g, flags=flags, dist_rd=dist_rd, dist_rs=dist_rs,

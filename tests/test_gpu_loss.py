@@ -344,3 +344,20 @@ def test_invalid_arguments_raise_before_launch():
         big = torch.zeros((5, 16), device="cuda")
         occ.occ_decoupled_loss_fwd_bwd(big[:4], i, f, f, f, None, rd_lo=0.5, rd_hi=2, eps_low=0.2,
                                        eps_high=0.28, dlogits=big[1:5])
+
+
+@pytest.mark.parametrize("rd_weight", [1, 0])
+def test_open_band_roles_of_table5(rd_weight):
+    # Table 5's "PPO-EWMA" and "linear_prox" rows weight by r_2 without masking
+    # it (r_2 * M(r_1)): an open band [0, inf) keeps every token in band.  With
+    # rd_weight = 0 the same band gives plain M(r_1) on pi_old.  The heavy-tailed
+    # batch puts many tokens far outside any finite band, so r_d reaches the
+    # gradient with large weights.
+    b = make_loss_batch("heavytail_bf16_v151936", T=300, seed=3, device="cuda")
+    b.rd_lo, b.rd_hi = 0.0, float("inf")
+    st, o = _full_parity(b, rd_weight=rd_weight)
+    assert st.n_rd_out == 0 == o["n_rd_out"]
+    v = o["valid"]
+    assert np.all((o["flags"][v] & FLAG_IN_BAND) != 0)
+    if rd_weight:
+        assert np.max(o["r_d"][v]) > 2.0 or np.min(o["r_d"][v]) < 0.5  # weights far from 1

@@ -335,3 +335,29 @@ def test_thresholds_inclusive_at_the_exact_bound():
     out = token_terms(lth, lold, lold, np.array([1.0, -1.0]), None, p)
     assert out["r_s"][0] == up and out["r_s"][1] == lo
     assert np.all(out["mis"]) and out["n_clipped"] == 0
+
+
+def test_open_band_role_weights_by_the_total_ratio():
+    # Table 5, "PPO-EWMA" row: r_2 * M(r_1) with no mask on r_2 (band [0, inf)).
+    # With a clip interval too wide to bind, every token is active and its
+    # weight is r_d * r_s = pi_theta / mu_old (the total ratio of Sec. 3.2), so
+    # the token-mean loss is -sum(exp(log pi_theta - log mu) * A) / N, computed
+    # here straight from the inputs.
+    rng = np.random.default_rng(17)
+    T = 64
+    lt = rng.normal(-3.0, 1.0, T)
+    lo = lt + rng.normal(0.0, 0.1, T)
+    lm = lo + rng.normal(0.0, 1.5, T)       # r_d spread over two orders of magnitude
+    A = rng.normal(0.0, 1.0, T)
+    m = (rng.random(T) < 0.8).astype(np.uint8)
+    p = LossParams(rd_lo=0.0, rd_hi=float("inf"), eps_low=1.0, eps_high=1e9, rd_weight=1)
+    o = token_terms(lt, lo, lm, A, m, p)
+    v = m.astype(bool)
+    assert o["n_rd_out"] == 0 and o["n_active"] == o["n_valid"] == v.sum()
+    expect = -math.fsum(np.exp(lt[v] - lm[v]) * A[v]) / v.sum()
+    assert abs(o["loss"] - expect) <= 1e-12 * max(1.0, abs(expect))
+    # without the r_d weight (rd_weight = 0) the same tokens weigh r_s alone
+    o0 = token_terms(lt, lo, lm, A, m, LossParams(rd_lo=0.0, rd_hi=float("inf"), eps_low=1.0,
+                                                  eps_high=1e9, rd_weight=0))
+    expect0 = -math.fsum(np.exp(lt[v] - lo[v]) * A[v]) / v.sum()
+    assert abs(o0["loss"] - expect0) <= 1e-12 * max(1.0, abs(expect0))
