@@ -47,6 +47,14 @@ WORKLOADS = {
         T=65536, V=V_QWEN3, dtype=torch.bfloat16, z_std=3.0, peak=8.0, heavy_frac=0.0,
         heavy_peak=0.0, old_std=0.2, mu=("normal", 0.02), adv=("grpo", 0.3, 8),
         layout=("packed", 128, 64, 1024), band=(0.8, 1.25), eps=(0.2, 0.28)),
+    # The thresholds of the paper's snapshot runs (App. C, run snap1004_1003: band
+    # [1/1.004, 1.004], clip 0.003 on both sides), with old-policy and rollout
+    # noise small enough that both ratios straddle them; float32 logits, since a
+    # bf16 logit step (2^-6 at |z| ~ 3) is coarser than the thresholds.
+    "tight_f32_v151936": dict(
+        T=2048, V=V_QWEN3, dtype=torch.float32, z_std=3.0, peak=8.0, heavy_frac=0.0,
+        heavy_peak=0.0, old_std=0.003, mu=("normal", 0.003), adv=("grpo", 0.3, 8),
+        layout=("fixed", 128), band=(1.0 / 1.004, 1.004), eps=(0.003, 0.003)),
     "heavytail_bf16_v151936": dict(
         T=16384, V=V_QWEN3, dtype=torch.bfloat16, z_std=3.0, peak=8.0, heavy_frac=0.1,
         heavy_peak=20.0, old_std=0.2, mu=("t2", 0.1), adv=("normal",), layout=("none",),

@@ -79,7 +79,8 @@ def _fused(b, **kw):
 
 @pytest.mark.parametrize("name,T", [("tiny_f32_v4096", 256), ("grpo_bf16_v32000", 600),
                                     ("agentic_bf16_v151936", 300),
-                                    ("heavytail_bf16_v151936", 300)])
+                                    ("heavytail_bf16_v151936", 300),
+                                    ("tight_f32_v151936", 384)])
 @pytest.mark.parametrize("diag", [True, False])
 def test_fused_workloads(name, T, diag):
     b = make_loss_batch(name, T=T, seed=4, device="cuda")

@@ -361,3 +361,15 @@ def test_open_band_roles_of_table5(rd_weight):
     assert np.all((o["flags"][v] & FLAG_IN_BAND) != 0)
     if rd_weight:
         assert np.max(o["r_d"][v]) > 2.0 or np.min(o["r_d"][v]) < 0.5  # weights far from 1
+
+
+@pytest.mark.parametrize("rd_weight", [1, 0])
+def test_paper_snapshot_thresholds(rd_weight):
+    # App. C's snapshot runs use thresholds of a few 1e-3 (snap1004_1003: band
+    # [1/1.004, 1.004], clip 0.003).  At that scale the decisions must still be
+    # bit-exact away from the 1e-6 exemption, with a fifth of the tokens out of
+    # band and a tenth clipped.
+    b = make_loss_batch("tight_f32_v151936", T=512, seed=5, device="cuda")
+    st, o = _full_parity(b, rd_weight=rd_weight, n_dz_rows=32)
+    assert 0.05 * o["n_valid"] < o["n_rd_out"] < 0.5 * o["n_valid"]
+    assert 0.03 * o["n_valid"] < o["n_clipped"] < 0.5 * o["n_valid"]
