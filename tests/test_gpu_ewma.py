@@ -132,3 +132,46 @@ def test_full_size_7p6e9_sampled():
     occ.occ_ewma_update(tp, th, 0.99, st)
     torch.cuda.synchronize()
     _check_step(before, thv, tp[it].cpu().numpy(), 0.99, 0.01)
+
+
+def test_checkpoint_and_resume_reproduce_the_run():
+    # The EWMA state is caller-owned (the proximal buffer and the 40-byte state
+    # with w, the coefficients, the streak and the reset count): saving both
+    # to the host and restoring them resumes the App. B recursion and the
+    # Sec. 5.2 streak exactly where it stopped.
+    n = 1_000_003
+    rng = np.random.default_rng(9)
+    thetas = [torch.from_numpy(rng.normal(0, 0.02, n).astype(np.float32)).to("cuda")
+              for _ in range(5)]
+    # low ratios at steps 1-2 (a streak that spans the checkpoint after step 1)
+    # and at steps 3-4: resets at steps 2 and 4
+    ratios = [(90, 100), (40, 100), (45, 100), (30, 100), (20, 100)]
+    stats = [occ.new_loss_stats("cuda") for _ in ratios]
+    for s, (act, val) in zip(stats, ratios):
+        # stats with the given n_active / n_valid (layout of occ_loss_stats)
+        buf = np.zeros(64, dtype=np.uint8)
+        buf[16:24] = np.frombuffer(np.int64(val).tobytes(), np.uint8)   # n_valid
+        buf[40:48] = np.frombuffer(np.int64(act).tobytes(), np.uint8)   # n_active
+        s.copy_(torch.from_numpy(buf))
+    tp0 = thetas[0].clone()
+
+    def run(tp, st, steps):
+        for k in steps:
+            occ.occ_ewma_update(tp, thetas[k], 0.75, st, stats=stats[k], tau=0.5, min_streak=2)
+
+    tp, st = tp0.clone(), occ.new_ewma_state("cuda")
+    run(tp, st, range(5))
+    torch.cuda.synchronize()
+
+    tp2, st2 = tp0.clone(), occ.new_ewma_state("cuda")
+    run(tp2, st2, range(2))
+    ckpt = (tp2.cpu().clone(), st2.cpu().clone())      # checkpoint after two steps
+    run(tp2, st2, range(2, 4))                         # progress that is thrown away
+    tp3, st3 = ckpt[0].to("cuda"), ckpt[1].to("cuda")  # resume from the checkpoint
+    run(tp3, st3, range(2, 5))
+    torch.cuda.synchronize()
+    assert torch.equal(tp3, tp) and torch.equal(st3, st)
+    s = occ.decode_ewma_state(st)
+    assert s.n_resets == 2 and s.streak == 0
+    saved = occ.decode_ewma_state(ckpt[1])
+    assert saved.streak == 1 and saved.n_resets == 0   # the step-2 reset needs the saved streak
