@@ -186,7 +186,7 @@ occ_status occ_decoupled_loss_fwd_bwd(const void* logits, occ_dtype dt, int64_t 
  * float64; the old row of a dropped token (mask 0 or bad id) is not read.
  * Results equal the two-call sequence up to that float32 rounding of log pi_old.
  * Optionally, in the same pass and with no extra memory traffic, per-token
- * diagnostics of the proximal reference's lag (Sec. 5.2, App. D):
+ * diagnostics of the proximal reference's lag (Sec. 5.2, App. E):
  *   entropy_out[t] = H(pi_theta(.|t)) = lse - sum_v p_v z_v
  *   kl_out[t]      = KL(pi_old(.|t) || pi_theta(.|t))
  * (both 0 for dropped tokens).

@@ -24,7 +24,7 @@ ewma   -- R10: the revised PPO-EWMA proximal parameters (Eq. 5, App. B),
 proxies -- R12: the log-linear and arithmetic interpolation proxies of
           Table 1 / App. A that stand in for a missing pi_old.
 diagnostics -- R11: per-token entropy of pi_theta and KL(pi_old || pi_theta),
-          the reference-lag diagnostics (Sec. 5.2, App. D).
+          the reference-lag diagnostics (Sec. 5.2, App. E).
 rows   -- chunking / threading driver (no arithmetic of the method).
 
 Pins: every function here is pinned by ``tests/test_oracle_*.py`` against

@@ -2,7 +2,7 @@
 
 TEST INFRASTRUCTURE ONLY (see the package docstring).
 
-Sec. 5.2 and App. D describe the failure mode the revised PPO-EWMA guards
+Sec. 5.2, Sec. 6.5 and App. E describe the failure mode the revised PPO-EWMA guards
 against: the reference policy drifts away from the policies that generated
 recent rollouts (reference-policy lag), which shows up as a collapsing
 Train-Infer Mask.  Two per-token quantities measure that lag directly from

@@ -12,7 +12,7 @@ and the update is the plain EWMA of Table 1 (b = 1 - beta).
 Sec. 5.2 also sets beta ~ W/(W+2) for a staleness window W (center of mass of
 the history, App. B) and resets theta_prox <- theta^(t) when the Train-Infer
 Mask value rho_t (fraction of tokens active after masking and clipping) drops
-below tau.  App. D speaks of consecutive low-ratio streaks; the oracle counts
+below tau.  App. E speaks of consecutive low-ratio streaks; the oracle counts
 a streak and resets once it reaches ``min_streak`` (1 = reset on the first low
 step, the Sec. 5.2 rule).  A step with no valid tokens carries no evidence:
 the streak is left unchanged.

@@ -11,7 +11,7 @@
 // Diagnostics (optional, no extra HBM bytes): the entropy of pi_theta,
 // H = lse - E_p[z], and KL(pi_old || pi_theta) = E_{p_old}[z_old - z] -
 // lse_old + lse, which track the reference-policy lag that the revised
-// PPO-EWMA is built to limit (Sec. 5.2, App. D).
+// PPO-EWMA is built to limit (Sec. 5.2, Sec. 6.5, App. E).
 #include "occ_loss_common.cuh"
 
 namespace occ {

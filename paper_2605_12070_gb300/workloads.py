@@ -47,7 +47,7 @@ WORKLOADS = {
         T=65536, V=V_QWEN3, dtype=torch.bfloat16, z_std=3.0, peak=8.0, heavy_frac=0.0,
         heavy_peak=0.0, old_std=0.2, mu=("normal", 0.02), adv=("grpo", 0.3, 8),
         layout=("packed", 128, 64, 1024), band=(0.8, 1.25), eps=(0.2, 0.28)),
-    # The thresholds of the paper's snapshot runs (App. C, run snap1004_1003: band
+    # The thresholds of the paper's snapshot runs (App. D, run snap1004_1003: band
     # [1/1.004, 1.004], clip 0.003 on both sides), with old-policy and rollout
     # noise small enough that both ratios straddle them; float32 logits, since a
     # bf16 logit step (2^-6 at |z| ~ 3) is coarser than the thresholds.

@@ -365,7 +365,7 @@ def test_open_band_roles_of_table5(rd_weight):
 
 @pytest.mark.parametrize("rd_weight", [1, 0])
 def test_paper_snapshot_thresholds(rd_weight):
-    # App. C's snapshot runs use thresholds of a few 1e-3 (snap1004_1003: band
+    # The snapshot runs of Sec. 6.4 / App. D use thresholds of a few 1e-3 (snap1004_1003: band
     # [1/1.004, 1.004], clip 0.003).  At that scale the decisions must still be
     # bit-exact away from the 1e-6 exemption, with a fifth of the tokens out of
     # band and a tenth clipped.
