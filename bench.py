@@ -21,6 +21,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import subprocess
 import sys
 import tempfile
@@ -135,14 +136,24 @@ KERNEL_SOURCES = {
 }
 
 
+_CODE_TOKENS = re.compile(r'"(?:\\.|[^"\\\n])*"|//[^\n]*|/\*.*?\*/', re.S)
+
+
+def _code_only(src):
+    """C++/CUDA source with comments removed and whitespace runs collapsed
+    (string literals kept), so that a comment edit keeps a capture valid."""
+    src = _CODE_TOKENS.sub(lambda m: m.group(0) if m.group(0).startswith('"') else " ", src)
+    return " ".join(src.split())
+
+
 def kernel_source_hash(name):
-    """Hash of the sources a kernel is built from (its traffic capture stays
-    valid while they are unchanged)."""
+    """Hash of the code a kernel is built from, comments and layout aside (its
+    traffic capture stays valid while that code is unchanged)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2605_12070_gb300", "csrc")
     for f in KERNEL_SOURCES[name]:
-        with open(os.path.join(csrc, f), "rb") as fh:
-            h.update(f.encode() + fh.read())
+        with open(os.path.join(csrc, f)) as fh:
+            h.update(f.encode() + _code_only(fh.read()).encode())
     return h.hexdigest()[:16]
 
 
