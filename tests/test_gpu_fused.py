@@ -179,3 +179,28 @@ def test_fused_full_size_agentic_sampled():
     H, K = _oracle_diag(b, rows)
     assert np.abs(out["entropy"].cpu().numpy()[rows][v] - H[v]).max() <= DIAG_TOL
     assert np.abs(out["kl"].cpu().numpy()[rows][v] - K[v]).max() <= DIAG_TOL
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 65536 + 3])
+def test_fused_vocab_edges(V, dtype):
+    # rows shorter than one vector, one vector exactly, a ragged tail after the
+    # vector body, and rows longer than the shared-memory head (65539 bf16 = 128 KB)
+    g = torch.Generator(device="cuda").manual_seed(V)
+    T = 37
+    z = (torch.randn((T, V), generator=g, device="cuda") * 2.5).to(dtype)
+    zo = (z.float() + 0.3 * torch.randn((T, V), generator=g, device="cuda")).to(dtype)
+    ids = torch.randint(0, V, (T,), generator=g, device="cuda", dtype=torch.int32)
+    ids[0], ids[-1] = 0, V - 1
+    lo64, _ = logprob_rows(zo, ids, np.arange(T))
+    lmu = torch.from_numpy(fp32(lo64 + np.random.default_rng(V).normal(0, 0.3, T))).cuda()
+    b = LossBatch("edge", z, zo, ids, lmu, torch.randn(T, generator=g, device="cuda"),
+                  (torch.rand(T, generator=g, device="cuda") < 0.8).to(torch.uint8),
+                  rd_lo=0.7, rd_hi=1.4)
+    out = _fused(b, want_diagnostics=True)
+    _check_fused(b, out, rows_dz=np.arange(T))
+    if V == 1:  # a one-token vocabulary: log pi = 0, entropy 0, KL 0
+        v = b.mask.cpu().numpy().astype(bool)
+        assert np.all(np.abs(out["logp"].cpu().numpy()[v]) <= 1e-5)
+        assert np.all(np.abs(out["entropy"].cpu().numpy()[v]) <= 1e-6)
+        assert np.all(np.abs(out["kl"].cpu().numpy()[v]) <= 1e-6)
