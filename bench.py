@@ -576,107 +576,6 @@ def run_e2e(args, batch, theta, theta_prox, state, stats, loss_fn, world, dev):
             "overlap": "copies on a second stream; loss and EWMA kernels run under them"}
 
 
-def _anon_huge_bytes():
-    """Anonymous memory of this host backed by transparent huge pages."""
-    try:
-        with open("/proc/meminfo") as f:
-            for line in f:
-                if line.startswith("AnonHugePages:"):
-                    return int(line.split()[1]) * 1024
-    except OSError:
-        pass
-    return 0
-
-
-def _host_available_bytes():
-    try:
-        with open("/proc/meminfo") as f:
-            for line in f:
-                if line.startswith("MemAvailable:"):
-                    return int(line.split()[1]) * 1024
-    except OSError:
-        pass
-    return 0
-
-
-def run_e2e(args, batch, theta, theta_prox, state, stats, loss_fn, world, dev):
-    """Same step through the public API with the inputs in pinned HOST memory:
-    every step copies the logits, token arrays and the new actor parameters to
-    the device and reads the loss statistics back.
-
-    The host link, not HBM, bounds this number, so the copies run on their own
-    stream and the kernels hide behind them: a step's loss runs while its
-    parameters are still copying, and its EWMA update while the next step's
-    logits copy.  Events keep each device buffer from being overwritten before
-    the kernel that reads it has finished."""
-    import torch
-
-    from paper_2605_12070_gb300 import dp, occ
-    loss_inputs = [batch.z_old, batch.z_theta, batch.ids, batch.logp_mu, batch.adv, batch.mask]
-    dev_inputs = loss_inputs + [theta]
-    need = sum(t.numel() * t.element_size() for t in dev_inputs)
-    if _host_available_bytes() < 1.3 * need:
-        return {"value": None, "unit": "tokens/s",
-                "skipped": f"needs {need / 1e9:.0f} GB of pinned host memory, "
-                           f"{_host_available_bytes() / 1e9:.0f} GB available"}
-    # page-locked, huge-page backed: the host link's address translation over
-    # 70 GB of buffers is the difference between ~100 and ~165 GB/s on some hosts
-    huge0 = _anon_huge_bytes()
-    host = [occ.occ_host_alloc(tuple(t.shape), t.dtype) for t in dev_inputs]
-    for h, d in zip(host, dev_inputs):
-        h.copy_(d)
-    huge = _anon_huge_bytes() - huge0
-    stats_h = torch.empty(occ.LOSS_STATS_BYTES, dtype=torch.uint8, pin_memory=True)
-    stream = torch.cuda.current_stream(dev)
-    copy_stream = torch.cuda.Stream(dev)
-    loss_done = torch.cuda.Event()
-    ewma_done = torch.cuda.Event()
-    loss_done.record(stream)
-    ewma_done.record(stream)
-
-    def e2e_step():
-        inputs_in, theta_in = torch.cuda.Event(), torch.cuda.Event()
-        with torch.cuda.stream(copy_stream):
-            copy_stream.wait_event(loss_done)           # previous loss has read the logits
-            for h, d in zip(host[:-1], dev_inputs[:-1]):
-                d.copy_(h, non_blocking=True)
-            inputs_in.record(copy_stream)
-            copy_stream.wait_event(ewma_done)           # previous update has read theta
-            dev_inputs[-1].copy_(host[-1], non_blocking=True)
-            theta_in.record(copy_stream)
-        stream.wait_event(inputs_in)
-        loss_fn()
-        loss_done.record(stream)
-        if world > 1:
-            dp.allreduce_loss_stats(stats)
-        stream.wait_event(theta_in)
-        occ.occ_ewma_update(theta_prox, theta, EWMA_BETA, state, stats=stats, tau=args.tau)
-        ewma_done.record(stream)
-        stats_h.copy_(stats, non_blocking=True)
-
-    e2e_step()
-    torch.cuda.synchronize()
-    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    s.record(stream)
-    copy_stream.wait_event(s)
-    for _ in range(args.e2e_steps):
-        e2e_step()
-    e.record(stream)
-    torch.cuda.synchronize()
-    sec = s.elapsed_time(e) / 1e3 / args.e2e_steps
-    if world > 1:
-        t = torch.tensor([sec], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        sec = float(t.item())
-    occ.decode_loss_stats(stats_h)
-    return {"value": round(world * batch.T / sec, 1), "unit": "tokens/s",
-            "h2d_bytes_per_step": need, "d2h_bytes_per_step": occ.LOSS_STATS_BYTES,
-            "ms_per_step": round(sec * 1e3, 3), "steps": args.e2e_steps,
-            "h2d_gbs": round(need / sec / 1e9, 1), "host_buffers": "occ_host_alloc (huge pages)",
-            "host_huge_page_fraction": round(min(1.0, max(0.0, huge / need)), 3),
-            "overlap": "copies on a second stream; loss and EWMA kernels run under them"}
-
-
 def run_ewma_variants(args, dev):
     """Times the bf16 proximal buffer (nearest and stochastic rounding, fp32 and
     bf16 theta) on --ewma-n parameters and the pinned-host buffer on 2e9."""
