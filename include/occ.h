@@ -312,7 +312,8 @@ occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* stream);
  * end-to-end step.  This is host plumbing: the paper has no counterpart.
  *
  * occ_host_alloc maps `bytes` (rounded up to the host's transparent-huge-page
- * size) of anonymous memory starting on a huge-page boundary, advises the
+ * size; a buffer smaller than one huge page is rounded to the base page and
+ * gets base pages) of anonymous memory starting on that boundary, advises the
  * kernel to back it with huge pages and page-locks it with cudaHostRegister.
  * The buffer is an ordinary page-locked buffer for cudaMemcpyAsync and for
  * occ_ewma_update_host; huge pages only cut the host link's address

@@ -6,7 +6,8 @@
 // spends its time on address translation when the buffer is mapped with base
 // pages: cudaHostAlloc memory moved ~100-110 GB/s over a 70 GB working set on
 // one box, while the same bytes in huge pages moved ~165 GB/s.  occ_host_alloc
-// maps anonymous memory aligned to the transparent-huge-page size, asks the
+// maps anonymous memory aligned to the transparent-huge-page size (buffers
+// smaller than one huge page: to the base page), asks the
 // kernel for huge pages (madvise; a kernel that declines gives base pages and
 // the buffer still works) and pins it with cudaHostRegister, so device copies
 // from it are asynchronous DMA like those from cudaHostAlloc memory.
@@ -36,6 +37,13 @@ static size_t thp_size() {
 
 static size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Granule of a buffer of `bytes`: the huge-page size once the buffer fills at
+// least one huge page, else the base page (a small buffer gains nothing from
+// huge pages and would pin a whole one).
+static size_t granule(size_t bytes) {
+  return bytes >= thp_size() ? thp_size() : (size_t)sysconf(_SC_PAGESIZE);
+}
+
 }  // namespace occ
 
 using namespace occ;
@@ -45,10 +53,10 @@ extern "C" occ_status occ_host_alloc(size_t bytes, void** out) {
   if (!out) return fail(OCC_ERR_INVALID_ARG, "null output pointer");
   *out = nullptr;
   if (bytes == 0) return fail(OCC_ERR_INVALID_ARG, "bytes == 0");
-  const size_t align = thp_size();
+  const size_t align = granule(bytes);
   const size_t len = round_up(bytes, align);
   if (len < bytes || len + align < len) return fail(OCC_ERR_INVALID_ARG, "size overflow");
-  // over-map by one huge page and trim, so that the buffer starts on a boundary
+  // over-map by one granule and trim, so that the buffer starts on a boundary
   void* raw = mmap(nullptr, len + align, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
   if (raw == MAP_FAILED) return fail(OCC_ERR_INVALID_ARG, "mmap of %zu bytes failed", len + align);
   const uintptr_t base = (uintptr_t)raw;
@@ -76,9 +84,10 @@ extern "C" occ_status occ_host_free(void* ptr, size_t bytes) {
   clear_error();
   if (!ptr) return OCC_OK;
   if (bytes == 0) return fail(OCC_ERR_INVALID_ARG, "bytes == 0");
-  if ((uintptr_t)ptr % thp_size() != 0)
+  const size_t align = granule(bytes);
+  if ((uintptr_t)ptr % align != 0)
     return fail(OCC_ERR_INVALID_ARG, "pointer was not returned by occ_host_alloc");
-  const size_t len = round_up(bytes, thp_size());
+  const size_t len = round_up(bytes, align);
   const cudaError_t e = cudaHostUnregister(ptr);
   munmap(ptr, len);
   if (e != cudaSuccess) {
