@@ -1,6 +1,6 @@
 """K3 parity: occ_ewma_update against the float64 oracle (R10).
 
-Tolerance: the benchmark spec's 1e-6 relative, taken relative to the magnitude of the
+Tolerance: the parity bar's 1e-6 relative, taken relative to the magnitude of the
 two terms of the App. B update, |a theta_prox| + |b theta| (which equals the
 result's magnitude unless the terms cancel).  Resets and first steps from an
 empty history must reproduce theta bit for bit.

@@ -1,6 +1,6 @@
 """K1 parity: occ_token_logprob against the float64 oracle (R1).
 
-Tolerance: the benchmark spec's 2e-3 absolute on log-probabilities, plus a tight
+Tolerance: the parity bar's 2e-3 absolute on log-probabilities, plus a tight
 bound derived from the kernel's arithmetic (float32 terms, compensated
 merge, float64 epilogue, float32 output): |err| <= 1e-5.
 """

@@ -1,6 +1,6 @@
 """K0 + K2 parity: occ_decoupled_loss_fwd_bwd against the float64 oracle (R1..R9).
 
-Bars (the benchmark spec): mask and clip flags bit-exact except tokens whose oracle
+Parity bars: mask and clip flags bit-exact except tokens whose oracle
 log-ratio lies within 1e-6 of the deciding threshold; log-probabilities within
 2e-3 absolute (tight bound 1e-5); loss within 1e-4 relative; dlogits within
 3e-3 absolute.  The dlogits bound used here is tighter and derived from the
