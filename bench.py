@@ -237,6 +237,13 @@ def oracle_sample_times(batch, rows, n_params, threads):
     return t_rows, t_par
 
 
+# Oracle timing calls: tokens and EWMA elements per call, shared by the
+# cpu_baseline leg and the reference arm (small calls are dominated by the
+# thread pool and by numpy's per-array overhead).
+REF_SAMPLE_ROWS = 512
+REF_SAMPLE_PARAMS = 1 << 26
+
+
 def cpu_baseline(batch, n_params_full, seconds):
     """Times the oracle, as it stands, on growing row chunks of the batch and an
     EWMA sample until about `seconds` of CPU work, then scales to one step."""
@@ -249,13 +256,13 @@ def cpu_baseline(batch, n_params_full, seconds):
     order = rng.permutation(valid)
     t_rows = t_par = 0.0
     n_rows = n_par = 0
-    chunk = 4 * threads
+    chunk = REF_SAMPLE_ROWS  # the reference arm's per-step sample: both time the same calls
     while t_rows < 0.7 * seconds and n_rows < order.size:
         rows = np.sort(order[n_rows:n_rows + chunk])
         tr, _ = oracle_sample_times(batch, rows, 0, threads)
         t_rows += tr
         n_rows += rows.size
-    par_chunk = 1 << 24
+    par_chunk = REF_SAMPLE_PARAMS
     while t_par < 0.3 * seconds and n_par < (1 << 30):
         _, tp = oracle_sample_times(batch, np.zeros(0, dtype=np.int64), par_chunk, threads)
         t_par += tp
@@ -638,7 +645,7 @@ def run_reference(args, batch, world):
     threads = host_cores()
     rng = np.random.default_rng(1)
     valid = np.nonzero(batch.mask.cpu().numpy())[0]
-    rows_n, params_n = 32, 1 << 23
+    rows_n, params_n = REF_SAMPLE_ROWS, REF_SAMPLE_PARAMS
     tot_rows = tot_par = 0.0
     for k in range(args.warmup + args.steps):
         rows = np.sort(rng.choice(valid, size=rows_n, replace=False))
