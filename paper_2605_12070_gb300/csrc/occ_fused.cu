@@ -359,6 +359,8 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
   constexpr int VEC = Elem<Tin>::kVec;
   constexpr int kCW = Gm::kCW, kNC = Gm::kNC, kHead = Gm::kHead, kSlots = Gm::kSlots;
   constexpr uint32_t kChunk = Gm::kChunk;
+  constexpr int kPer = (int)(kChunk / 16) / kNC;  // vectors per consumer thread in a full chunk
+  static_assert(kPer * kNC * 16 == (int)kChunk, "a chunk splits evenly over the consumers");
   extern __shared__ __align__(128) unsigned char ring_smem[];
   __shared__ Shared<Gm::kCW, Gm::kHead, Gm::kSlots> sh;
   const K2Args& a = f.a;
@@ -514,12 +516,30 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
       ++G;
       if (!ok) break;
       const uint4* os = reinterpret_cast<const uint4*>(slots + (size_t)so * kChunk);
-      for (int i = ct; i < nv; i += kNC) {
+      auto fwd = [&](int i) {
         float x[VEC], xo[VEC];
         Elem<Tin>::unpack(zs[i], x);
         accv_add<VEC, false>(acc[0], x, x);
         Elem<Tin>::unpack(os[i], xo);
         accv_add<VEC, false>(acc[1], xo, xo);
+      };
+      if (nv == kPer * kNC) {  // a full chunk: straight-line, compile-time trip count
+        uint4 rz[kPer], ro[kPer];
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) {
+          rz[u] = zs[ct + u * kNC];
+          ro[u] = os[ct + u * kNC];
+        }
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) {
+          float x[VEC], xo[VEC];
+          Elem<Tin>::unpack(rz[u], x);
+          accv_add<VEC, false>(acc[0], x, x);
+          Elem<Tin>::unpack(ro[u], xo);
+          accv_add<VEC, false>(acc[1], xo, xo);
+        }
+      } else {
+        for (int i = ct; i < nv; i += kNC) fwd(i);
       }
       __syncwarp();
       if (lane == 0) {
@@ -589,18 +609,26 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
       }
       OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
     };
+    auto bwd_chunk = [&](const uint4* zs, int64_t base, int nv) {
+      if (g == 0.f) {
+        for (int i = ct; i < nv; i += kNC) OutVecHint<Tout, VEC>::zero(drow + (base + i) * VEC, last);
+      } else if (nv == kPer * kNC) {
+        uint4 r[kPer];
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) r[u] = zs[ct + u * kNC];
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) emit(base + ct + u * kNC, r[u]);
+      } else {
+        for (int i = ct; i < nv; i += kNC) emit(base + i, zs[i]);
+      }
+    };
     // backward: the head from shared memory, then the re-read chunks
     if (drow) {
       for (int k = 0; k < nhead; ++k) {
         const int nv = (int)(chunk_bytes(k) / 16);
         const uint4* zs = reinterpret_cast<const uint4*>(head + (size_t)k * kChunk);
         const int64_t base = (int64_t)k * (kChunk / 16);
-        for (int i = ct; i < nv; i += kNC) {
-          if (g == 0.f)
-            OutVecHint<Tout, VEC>::zero(drow + (base + i) * VEC, last);
-          else
-            emit(base + i, zs[i]);
-        }
+        bwd_chunk(zs, base, nv);
       }
     }
     __syncwarp();
@@ -614,12 +642,7 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
         if (!ok) break;
         const uint4* zs = reinterpret_cast<const uint4*>(slots + (size_t)s * kChunk);
         const int64_t base = (int64_t)k * (kChunk / 16);
-        for (int i = ct; i < nv; i += kNC) {
-          if (g == 0.f)
-            OutVecHint<Tout, VEC>::zero(drow + (base + i) * VEC, last);
-          else
-            emit(base + i, zs[i]);
-        }
+        bwd_chunk(zs, base, nv);
         __syncwarp();
         if (lane == 0) arrive(&sh.empty[s]);
       }
