@@ -131,7 +131,8 @@ class ClockSampler:
 KERNEL_SOURCES = {
     "k1_token_logprob": ("occ_logprob.cu", "occ_common.cuh"),
     "k2_decoupled_loss_fwd_bwd": ("occ_loss.cu", "occ_loss_common.cuh", "occ_common.cuh"),
-    "k12_decoupled_loss_fused": ("occ_fused.cu", "occ_loss_common.cuh", "occ_common.cuh"),
+    "k12_decoupled_loss_fused": ("occ_fused.cu", "occ_fused_common.cuh", "occ_loss_common.cuh",
+                                 "occ_common.cuh"),
     "k3_ewma_update": ("occ_ewma.cu", "occ_common.cuh"),
 }
 
