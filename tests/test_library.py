@@ -101,3 +101,38 @@ def test_host_alloc_fails_cleanly_without_a_device(L):
     p = ctypes.c_void_p()
     assert L.occ_host_alloc(1 << 20, ctypes.byref(p)) == 4  # OCC_ERR_CUDA
     assert p.value is None and b"cudaHostRegister" in L.occ_last_error()
+
+
+def test_error_messages_are_per_host_thread(L):
+    # occ_last_error is documented per host thread: a failing call in one
+    # thread must not overwrite the message another thread is about to read.
+    import threading
+    null = ctypes.c_void_p(0)
+    st = ctypes.create_string_buffer(48)
+    stp = ctypes.cast(st, ctypes.c_void_p)
+    barrier = threading.Barrier(2)
+    seen = {}
+
+    def logprob_thread():
+        for _ in range(200):
+            assert L.occ_token_logprob(null, 0, 4, 0, 0, null, null, null, null) == 1
+            barrier.wait()
+            msg = L.occ_last_error()
+            barrier.wait()
+            seen.setdefault("logprob", set()).add(msg)
+
+    def ewma_thread():
+        for _ in range(200):
+            assert L.occ_ewma_update(null, null, 0, 1.5, stp, null, 0.9, 1, 0, null) == 1
+            barrier.wait()
+            msg = L.occ_last_error()
+            barrier.wait()
+            seen.setdefault("ewma", set()).add(msg)
+
+    ts = [threading.Thread(target=logprob_thread), threading.Thread(target=ewma_thread)]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join()
+    assert len(seen["logprob"]) == 1 and b"V >= 1" in next(iter(seen["logprob"]))
+    assert len(seen["ewma"]) == 1 and b"beta" in next(iter(seen["ewma"]))
