@@ -50,11 +50,12 @@ WORKLOADS = {
     # The thresholds of the paper's snapshot runs (App. D, run snap1004_1003: band
     # [1/1.004, 1.004], clip 0.003 on both sides), with old-policy and rollout
     # noise small enough that both ratios straddle them; float32 logits, since a
-    # bf16 logit step (2^-6 at |z| ~ 3) is coarser than the thresholds.
+    # bf16 logit step (2^-6 at |z| ~ 3) is coarser than the thresholds; per-token
+    # N(0, 1) advantages of both signs, so every token carries a gradient.
     "tight_f32_v151936": dict(
         T=2048, V=V_QWEN3, dtype=torch.float32, z_std=3.0, peak=8.0, heavy_frac=0.0,
-        heavy_peak=0.0, old_std=0.003, mu=("normal", 0.003), adv=("grpo", 0.3, 8),
-        layout=("fixed", 128), band=(1.0 / 1.004, 1.004), eps=(0.003, 0.003)),
+        heavy_peak=0.0, old_std=0.003, mu=("normal", 0.003), adv=("normal",),
+        layout=("none",), band=(1.0 / 1.004, 1.004), eps=(0.003, 0.003)),
     "heavytail_bf16_v151936": dict(
         T=16384, V=V_QWEN3, dtype=torch.bfloat16, z_std=3.0, peak=8.0, heavy_frac=0.1,
         heavy_peak=20.0, old_std=0.2, mu=("t2", 0.1), adv=("normal",), layout=("none",),
@@ -107,7 +108,11 @@ def _sequence_layout(spec, rng, T):
     adv = np.zeros(T, dtype=np.float32)
     mask = None
     if kind == "fixed":
+        # a batch resized below the workload's T keeps its number of sequences
+        # (shorter ones), so that its GRPO groups still have spread advantages
         L = spec["layout"][1]
+        if T < spec["T"]:
+            L = max(1, (L * T) // spec["T"])
         n_seq = (T + L - 1) // L
         A = _grpo_advantages(rng, n_seq, spec["adv"][1], spec["adv"][2])
         adv[:] = np.repeat(A, L)[:T]

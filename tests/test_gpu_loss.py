@@ -373,3 +373,4 @@ def test_paper_snapshot_thresholds(rd_weight):
     st, o = _full_parity(b, rd_weight=rd_weight, n_dz_rows=32)
     assert 0.05 * o["n_valid"] < o["n_rd_out"] < 0.5 * o["n_valid"]
     assert 0.03 * o["n_valid"] < o["n_clipped"] < 0.5 * o["n_valid"]
+    assert np.count_nonzero(o["g"]) > 0.3 * o["n_valid"]   # the dlogits check is not vacuous
