@@ -29,7 +29,7 @@ def _oracle_diag(b, rows):
     return orc.token_entropy(z), orc.token_kl(zo, z)
 
 
-def _check_fused(b, out, rows_dz=None, f32=False, diag=True):
+def _check_fused(b, out, rows_dz=None, f32=False, diag=True, require_grad=True):
     T = b.T
     rows = np.arange(T)
     lo64, _ = logprob_rows(b.z_old, b.ids, rows)
@@ -60,6 +60,8 @@ def _check_fused(b, out, rows_dz=None, f32=False, diag=True):
         act = np.nonzero(o["g"] != 0)[0]
         rows_dz = np.unique(np.concatenate([act[:24], [0, T - 1]]))
     rows_dz = np.array([r for r in rows_dz if not diff[r]], dtype=np.int64)
+    if require_grad and o["n_valid"] > 0:  # the batch must exercise the gradient
+        assert np.count_nonzero(o["g"][rows_dz]) > 0, "no compared row carries a gradient"
     ref = dlogits_rows(b, rows_dz, lse[rows_dz], o["g"][rows_dz])
     got = out["dlogits"][torch.as_tensor(rows_dz, device="cuda")].float().cpu().numpy()
     g = np.abs(o["g"][rows_dz])[:, None]

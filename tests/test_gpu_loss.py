@@ -104,6 +104,8 @@ def _full_parity(batch, rd_weight=1, dlogits_f32=False, grad_scale=1.0, n_dz_row
         pick += list(rng.choice(act, size=min(n_dz_rows, act.size), replace=False))
     pick += list(rng.choice(T, size=min(8, T), replace=False))
     dz_rows = np.unique(np.array(pick))
+    if o["n_valid"] > 0:  # the batch must exercise the gradient, not compare zeros
+        assert np.count_nonzero(o["g"][dz_rows]) > 0, "no compared row carries a gradient"
     return _compare(batch, out, o, lp_th64, dz_rows=dz_rows, lse=lse_th[dz_rows],
                     out_f32=dlogits_f32 or batch.z_theta.dtype == torch.float32), o
 
