@@ -136,3 +136,18 @@ def test_error_messages_are_per_host_thread(L):
         t.join()
     assert len(seen["logprob"]) == 1 and b"V >= 1" in next(iter(seen["logprob"]))
     assert len(seen["ewma"]) == 1 and b"beta" in next(iter(seen["ewma"]))
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    # without libocc.so every entry point raises; nothing falls back to a CPU path
+    import torch
+    monkeypatch.setattr(occ, "LIB_PATH", str(tmp_path / "libocc.so"))
+    monkeypatch.setattr(occ, "_lib", None)
+    with pytest.raises(occ.OccError, match="not built"):
+        occ.lib()
+    with pytest.raises(occ.OccError):
+        occ.occ_loss_workspace_bytes(16, 32)
+    if torch.cuda.is_available():
+        with pytest.raises(occ.OccError, match="not built"):
+            occ.occ_token_logprob(torch.zeros(2, 4, device="cuda"),
+                                  torch.zeros(2, dtype=torch.int32, device="cuda"))
