@@ -540,10 +540,19 @@ def run_e2e(args, batch, theta, theta_prox, state, stats, loss_fn, world, dev):
     from paper_2605_12070_gb300.pipeline import HostFedStep
     loss_inputs = [batch.z_old, batch.z_theta, batch.ids, batch.logp_mu, batch.adv, batch.mask]
     need = sum(t.numel() * t.element_size() for t in loss_inputs + [theta])
-    if _host_available_bytes() < 1.3 * need:
+    # every rank on this host pins its own copy: check for all of them at once,
+    # after a barrier so that no rank has allocated yet, and decide together
+    local = int(os.environ.get("LOCAL_WORLD_SIZE", str(world)))
+    if world > 1:
+        torch.distributed.barrier()
+    avail = _host_available_bytes()
+    fits = torch.tensor([1 if avail >= 1.3 * need * local else 0], device=dev)
+    if world > 1:
+        torch.distributed.all_reduce(fits, op=torch.distributed.ReduceOp.MIN)
+    if not int(fits.item()):
         return {"value": None, "unit": "tokens/s",
-                "skipped": f"needs {need / 1e9:.0f} GB of pinned host memory, "
-                           f"{_host_available_bytes() / 1e9:.0f} GB available"}
+                "skipped": f"needs {local} x {need / 1e9:.0f} GB of pinned host memory, "
+                           f"{avail / 1e9:.0f} GB available"}
     # page-locked, huge-page backed: the host link's address translation over
     # 70 GB of buffers is the difference between ~100 and ~165 GB/s on some hosts
     huge0 = _anon_huge_bytes()
