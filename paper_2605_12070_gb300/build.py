@@ -6,6 +6,7 @@ so the library loads without a GPU and the only driver dependency is resolved
 when the first CUDA call runs.  Usage: ``python -m paper_2605_12070_gb300.build``.
 """
 
+import fcntl
 import os
 import subprocess
 import sys
@@ -44,8 +45,21 @@ def _compile(src, verbose):
 
 
 def build(verbose=False, force=False):
-    """Compiles every .cu under csrc/ and links libocc.so.  Returns the library path."""
+    """Compiles every .cu under csrc/ and links libocc.so.  Returns the library path.
+
+    Processes that build at the same time (ranks of one job, parallel tests)
+    take turns on a lock file: the first compiles, the others then find the
+    library up to date."""
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            return _build_locked(verbose, force)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose, force):
     srcs = sources()
     deps = srcs + [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))]
     deps += [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE)]

@@ -151,3 +151,21 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
         with pytest.raises(occ.OccError, match="not built"):
             occ.occ_token_logprob(torch.zeros(2, 4, device="cuda"),
                                   torch.zeros(2, dtype=torch.int32, device="cuda"))
+
+
+def test_concurrent_builds_take_turns():
+    # ranks of one job (or parallel test workers) may all call build(): one
+    # forced rebuild and two plain ones at the same time must all succeed and
+    # leave a library that exports every entry point
+    import subprocess
+    import sys
+    code = "from paper_2605_12070_gb300 import build; build.build(force={})"
+    procs = [subprocess.Popen([sys.executable, "-c", code.format(f)], cwd=ROOT,
+                              stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True)
+             for f in (True, False, False)]
+    for p in procs:
+        out, err = p.communicate(timeout=900)
+        assert p.returncode == 0, err[-2000:]
+    L2 = ctypes.CDLL(build.LIB)
+    for name in occ.EXPORTS:
+        assert hasattr(L2, name), name
