@@ -239,10 +239,27 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
   if (vec && !DIAG && f.a.V >= Elem<Tin>::kVec && fused_ring_selected())
     return launch_fused_ring<Tin, Tout>(f, s);
   if (vec) {
+    static const int nt_env = [] {
+      const char* e = getenv("OCC_FUSED_THREADS");
+      return e ? atoi(e) : 0;
+    }();
+    static const long head_env = [] {
+      const char* e = getenv("OCC_FUSED_HEAD_KB");
+      return e ? atol(e) * 1024 : -1L;
+    }();
+    // Row-size tiers (measured on GB300, V = 32000 to 151936 bf16): short rows
+    // finish in about one load round per CTA, so small CTAs, more of them per
+    // SM and no shared-memory head (L2 holds every row in flight) keep the
+    // memory system busy; long rows want 512 threads and the 80 KB head.
     const size_t row_bytes = (size_t)(f.a.V / Elem<Tin>::kVec) * 16;
-    const size_t head = std::min(kFusedHeadBytes, row_bytes);
+    const int nt_auto = row_bytes <= 64 * 1024 ? 128 : row_bytes <= 112 * 1024 ? 256 : kFusedThreads;
+    const int nt = nt_env ? nt_env : nt_auto;
+    const size_t head_auto = nt_auto == kFusedThreads ? kFusedHeadBytes : 0;
+    const size_t head = std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
     f.a.stage_bytes = (int64_t)head;
-    auto kern = k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, DIAG>;
+    auto kern = nt == 128   ? k2_fused_l2<Tin, Tout, 128, kFusedUnroll, DIAG>
+                : nt == 256 ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, DIAG>
+                            : k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, DIAG>;
     if (head > 0) {
       cudaError_t e =
           cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)head);
@@ -252,7 +269,7 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
     }
     for (int64_t r0 = 0; r0 < T; r0 += step) {
       f.a.row0 = r0;
-      kern<<<(unsigned)std::min<int64_t>(step, T - r0), kFusedThreads, head, s>>>(f);
+      kern<<<(unsigned)std::min<int64_t>(step, T - r0), nt, head, s>>>(f);
     }
   } else {
     for (int64_t r0 = 0; r0 < T; r0 += step) {

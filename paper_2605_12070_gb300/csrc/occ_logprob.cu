@@ -6,6 +6,8 @@
 // U vectors in flight per thread, and keeps an online (c, s) pair per thread;
 // nothing is staged in shared memory because each element is used once.
 // HBM traffic is the logits row once: V * sizeof(T) bytes per token.
+#include <cstdlib>
+
 #include "occ_common.cuh"
 
 namespace occ {
@@ -14,7 +16,7 @@ constexpr int kK1Threads = 512;
 constexpr int kK1Unroll = 8;
 
 template <typename Tin, int NT, int U>
-__global__ void __launch_bounds__(NT, 2)
+__global__ void __launch_bounds__(NT, 1024 / NT)
     k1_logprob_vec(const Tin* __restrict__ logits, int64_t T, int64_t V, int64_t ld,
                    const int32_t* __restrict__ ids, float* __restrict__ logp,
                    float* __restrict__ lse_out) {
@@ -108,10 +110,25 @@ template <typename Tin>
 static void launch_k1(const void* logits, int64_t T, int64_t V, int64_t ld, const int32_t* ids,
                       float* logp, float* lse, bool vec, cudaStream_t s) {
   const unsigned grid = (unsigned)(T < 0x7fffffffLL ? T : 0x7fffffffLL);
-  if (vec)
-    k1_logprob_vec<Tin, kK1Threads, kK1Unroll><<<grid, kK1Threads, 0, s>>>(
-        (const Tin*)logits, T, V, ld, ids, logp, lse);
-  else
+  static const int nt_env = [] {
+    const char* e = getenv("OCC_K1_THREADS");
+    return e ? atoi(e) : 0;
+  }();
+  if (vec) {
+    // rows up to ~96 KB: 128 threads; longer rows: 256 (measured on GB300 from
+    // V = 32000 to 151936 bf16; 512 threads left 2-50 % on the table)
+    const int64_t row_bytes = (V / Elem<Tin>::kVec) * 16;
+    const int nt = nt_env ? nt_env : (row_bytes <= 96 * 1024 ? 128 : 256);
+    if (nt == 128)
+      k1_logprob_vec<Tin, 128, kK1Unroll><<<grid, 128, 0, s>>>((const Tin*)logits, T, V, ld, ids,
+                                                              logp, lse);
+    else if (nt == 256)
+      k1_logprob_vec<Tin, 256, kK1Unroll><<<grid, 256, 0, s>>>((const Tin*)logits, T, V, ld, ids,
+                                                              logp, lse);
+    else
+      k1_logprob_vec<Tin, kK1Threads, kK1Unroll><<<grid, kK1Threads, 0, s>>>(
+          (const Tin*)logits, T, V, ld, ids, logp, lse);
+  } else
     k1_logprob_scalar<Tin, kK1Threads><<<grid, kK1Threads, 0, s>>>((const Tin*)logits, T, V, ld,
                                                                     ids, logp, lse);
 }

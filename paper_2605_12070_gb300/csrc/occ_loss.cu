@@ -917,22 +917,35 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
         return launch_persistent(k2_loss_tma<Tin, Tout, 256, kK2Stages>, 256, a, pl, kK2Stages, s);
       }
     }
-    // shared-memory row head: OCC_K2_HEAD_KB overrides (0 = pure L2 re-read)
-    static const size_t head_cap = [] {
-      const char* e = getenv("OCC_K2_HEAD_KB");
-      return (size_t)(e ? atoi(e) : 80) * 1024;
-    }();
+    // Row-size tiers (measured on GB300, V = 32000 to 151936 bf16): 128 threads
+    // and a 16 KB head up to 64 KB rows, 256 threads and no head up to 112 KB,
+    // 512 threads and an 80 KB head beyond.  OCC_K2_L2_THREADS and
+    // OCC_K2_HEAD_KB override (0 = pure L2 re-read).
     const size_t row_bytes = (size_t)(a.V / Elem<Tin>::kVec) * 16;
-    const size_t head_bytes = std::min(head_cap, row_bytes);
+    const int nt_auto = row_bytes <= 64 * 1024 ? 128 : row_bytes <= 112 * 1024 ? 256 : 512;
+    static const long head_env = [] {
+      const char* e = getenv("OCC_K2_HEAD_KB");
+      return e ? atol(e) * 1024 : -1L;
+    }();
+    const size_t head_auto = nt_auto == 128 ? 16 * 1024 : nt_auto == 256 ? 0 : 80 * 1024;
+    const size_t head_bytes =
+        std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
     a.stage_bytes = (int64_t)head_bytes;
     static const int unroll = [] {
       const char* e = getenv("OCC_K2_UNROLL");
       return e ? atoi(e) : 8;
     }();
-    auto kern = (var == 3) ? k2_loss_l2<Tin, Tout, 1024, 8>
-                           : (unroll == 4 ? k2_loss_l2<Tin, Tout, 512, 4>
-                                          : k2_loss_l2<Tin, Tout, 512, 8>);
-    const int nt = (var == 3) ? 1024 : 512;
+    static const int nt_env = [] {
+      const char* e = getenv("OCC_K2_L2_THREADS");
+      return e ? atoi(e) : 0;
+    }();
+    const int nt_small = nt_env ? nt_env : nt_auto;
+    auto kern = (var == 3)            ? k2_loss_l2<Tin, Tout, 1024, 8>
+                : (nt_small == 128) ? k2_loss_l2<Tin, Tout, 128, 8>
+                : (nt_small == 256) ? k2_loss_l2<Tin, Tout, 256, 8>
+                : (unroll == 4)       ? k2_loss_l2<Tin, Tout, 512, 4>
+                                      : k2_loss_l2<Tin, Tout, 512, 8>;
+    const int nt = (var == 3) ? 1024 : (nt_small == 128 || nt_small == 256) ? nt_small : 512;
     if (head_bytes > 0) {
       cudaError_t e =
           cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)head_bytes);
