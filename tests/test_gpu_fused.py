@@ -184,10 +184,11 @@ def test_fused_full_size_agentic_sampled():
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 65536 + 3])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 20000, 50000, 65536 + 3])
 def test_fused_vocab_edges(V, dtype):
     # rows shorter than one vector, one vector exactly, a ragged tail after the
-    # vector body, and rows longer than the shared-memory head (65539 bf16 = 128 KB)
+    # vector body, rows in each CTA-size tier (40 / 80 / 100 / 200 KB) and rows
+    # longer than the shared-memory head (65539 bf16 = 128 KB)
     g = torch.Generator(device="cuda").manual_seed(V)
     T = 37
     z = (torch.randn((T, V), generator=g, device="cuda") * 2.5).to(dtype)

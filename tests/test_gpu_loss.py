@@ -225,7 +225,7 @@ def _edge_batch(T, V, dtype, seed, mask_p=0.8, ld=None, offset=0):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 65536 + 3])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 20000, 50000, 65536 + 3])
 def test_vocab_edges(V, dtype):
     T = 37
     b, lp_old64 = _edge_batch(T, V, dtype, seed=V)
