@@ -51,6 +51,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--tau", type=float, default=0.5)
     ap.add_argument("--tokens", type=int, default=None, help="resize T (profiling runs only)")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="loss batch (default: the agentic batch the metric is quoted on; the "
+                         "others are for breakdowns only)")
     ap.add_argument("--ewma-variants", action="store_true",
                     help="instead of the step, time the bf16 and host-resident EWMA buffers")
     ap.add_argument("--loss-path", default="fused", choices=["fused", "two-call"],
@@ -301,9 +304,9 @@ def main():
     from paper_2605_12070_gb300 import dp, occ
     from paper_2605_12070_gb300.workloads import make_ewma_buffers, make_loss_batch
 
-    batch = make_loss_batch(WORKLOAD, T=args.tokens, seed=rank, device=dev)
+    batch = make_loss_batch(args.workload, T=args.tokens, seed=rank, device=dev)
     T, V = batch.T, batch.V
-    n_valid = int(batch.mask.sum().item())
+    n_valid = T if batch.mask is None else int(batch.mask.sum().item())
 
     if args.impl == "reference":
         run_reference(args, batch, world)
@@ -316,7 +319,7 @@ def main():
     theta, theta_prox = make_ewma_buffers(args.ewma_n, seed=rank, device=dev)
     state = occ.new_ewma_state(dev, w0=1.0 / (1.0 - EWMA_BETA))
     lp_old = torch.empty(T, dtype=torch.float32, device=dev)
-    dlogits = torch.empty((T, V), dtype=torch.bfloat16, device=dev)
+    dlogits = torch.empty((T, V), dtype=batch.z_theta.dtype, device=dev)
     logp = torch.empty(T, dtype=torch.float32, device=dev)
     flags = torch.empty(T, dtype=torch.uint8, device=dev)
     stats = occ.new_loss_stats(dev)
@@ -426,9 +429,10 @@ def main():
 
     peak, peak_kind = measured_peak()
     traffic = ncu_traffic()
-    bytes_k1 = T * V * 2 + T * 8
-    bytes_k2 = n_valid * V * 2 + T * V * 2 + T * 37
-    bytes_fused = 2 * n_valid * V * 2 + T * V * 2 + T * 41
+    es = batch.z_theta.element_size()
+    bytes_k1 = T * V * es + T * 8
+    bytes_k2 = n_valid * V * es + T * V * es + T * 37
+    bytes_fused = 2 * n_valid * V * es + T * V * es + T * 41
     # a regular update reads theta_prox and theta and writes theta_prox; a reset copies theta
     bytes_k3 = args.ewma_n * (12 * (args.steps - resets) + 8 * resets) // args.steps
     st_last = occ.decode_loss_stats(stats)
@@ -472,14 +476,16 @@ def main():
         "dtype": "f32",
         "data": "synthetic",
         "config": {
-            "workload": (f"decoupled-loss step on T={T} tokens (128 packed sequences, "
-                         f"{n_valid} valid), V={V} bf16 old and current logits (log pi_old, "
-                         f"loss fwd + dlogits) chained with the PPO-EWMA update of "
-                         f"{args.ewma_n} fp32 parameters"),
+            "workload": (f"decoupled-loss step on the {args.workload} batch, T={T} tokens "
+                         f"({n_valid} valid), V={V} {str(batch.z_theta.dtype).replace('torch.', '')} "
+                         f"old and current logits (log pi_old, loss fwd + dlogits) chained with the "
+                         f"PPO-EWMA update of {args.ewma_n} fp32 parameters"),
             "loss_path": args.loss_path,
-            "T": T, "V": V, "ewma_params": args.ewma_n, "logits_dtype": "bf16",
+            "T": T, "V": V, "ewma_params": args.ewma_n,
+            "logits_dtype": str(batch.z_theta.dtype).replace("torch.", ""),
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-            "l2": "inputs larger than L2 (40 GB logits, 61 GB EWMA buffers): no flush",
+            "l2": (f"inputs larger than L2 ({2 * T * V * es / 1e9:.0f} GB logits, "
+                   f"{8 * args.ewma_n / 1e9:.0f} GB EWMA buffers): no flush"),
             "rd_band": [batch.rd_lo, batch.rd_hi], "eps": [batch.eps_low, batch.eps_high],
             "tau": args.tau, "rho": round(st_last.rho, 5), "ewma_resets_timed": resets,
         },
@@ -538,7 +544,9 @@ def run_e2e(args, batch, theta, theta_prox, state, stats, loss_fn, world, dev):
 
     from paper_2605_12070_gb300 import dp, occ
     from paper_2605_12070_gb300.pipeline import HostFedStep
-    loss_inputs = [batch.z_old, batch.z_theta, batch.ids, batch.logp_mu, batch.adv, batch.mask]
+    loss_inputs = [batch.z_old, batch.z_theta, batch.ids, batch.logp_mu, batch.adv]
+    if batch.mask is not None:
+        loss_inputs.append(batch.mask)
     need = sum(t.numel() * t.element_size() for t in loss_inputs + [theta])
     # every rank on this host pins its own copy: check for all of them at once,
     # after a barrier so that no rank has allocated yet, and decide together
@@ -654,8 +662,9 @@ def run_reference(args, batch, world):
     from oracle.rows import host_cores
     threads = host_cores()
     rng = np.random.default_rng(1)
-    valid = np.nonzero(batch.mask.cpu().numpy())[0]
-    rows_n, params_n = REF_SAMPLE_ROWS, REF_SAMPLE_PARAMS
+    valid = (np.arange(batch.T) if batch.mask is None
+             else np.nonzero(batch.mask.cpu().numpy())[0])
+    rows_n, params_n = min(REF_SAMPLE_ROWS, valid.size), REF_SAMPLE_PARAMS
     tot_rows = tot_par = 0.0
     for k in range(args.warmup + args.steps):
         rows = np.sort(rng.choice(valid, size=rows_n, replace=False))
