@@ -27,8 +27,14 @@
  *     occ_loss_stats.err.
  *   - Logits are row-major [T, V] with a row stride `ld` >= V elements.
  *     Rows whose start is 16-byte aligned (base address and ld * element size
- *     multiples of 16) use the vectorised kernels; any other layout runs on a
- *     scalar-load kernel of the same library, with identical results.
+ *     multiples of 16) use the vectorised kernels.  Rows off that boundary
+ *     run the same kernels peeled (scalar loads up to the boundary, then
+ *     16-byte loads) when every other row array of the call (old logits,
+ *     dlogits) has the same element size and sits at the same byte offsets
+ *     (base addresses and row strides congruent modulo 16 bytes) and
+ *     V >= 128 (bf16) / 64 (f32); any other layout runs on a scalar-load
+ *     kernel.  All three meet the same accuracy bounds; occ_last_kernel()
+ *     names the one a call took.
  */
 #ifndef OCC_H_
 #define OCC_H_
@@ -336,6 +342,16 @@ const char* occ_status_string(occ_status s);
 
 /* Message of the last failed call on this host thread ("" if none). */
 const char* occ_last_error(void);
+
+/* The row kernel that the last call on this host thread launched, as a static
+ * string: "k1_logprob_vec", "k1_logprob_vec/peel", "k1_logprob_scalar",
+ * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_stream", "k2_loss_tma",
+ * "k2_loss_reg", "k2_fused_l2", "k2_fused_l2/peel", "k2_fused_stream",
+ * "k2_fused_ring", "k3_ewma_vec", "k3_ewma_scalar", "k3_ewma_bf16" ("" when
+ * the call launched none, e.g. T = 0 or an invalid argument).  "/peel" marks
+ * the vector kernel run on rows that start off a 16-byte boundary.  Never
+ * freed; valid until the next call on the thread. */
+const char* occ_last_kernel(void);
 
 /* OCC_VERSION of the built library. */
 int occ_version(void);

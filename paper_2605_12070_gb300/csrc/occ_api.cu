@@ -7,6 +7,7 @@
 namespace occ {
 
 static thread_local char g_msg[512] = "";
+static thread_local const char* g_kernel = "";
 
 occ_status fail(occ_status s, const char* fmt, ...) {
   va_list ap;
@@ -16,7 +17,12 @@ occ_status fail(occ_status s, const char* fmt, ...) {
   return s;
 }
 
-void clear_error() { g_msg[0] = '\0'; }
+void clear_error() {
+  g_msg[0] = '\0';
+  g_kernel = "";
+}
+
+void note_kernel(const char* name) { g_kernel = name; }
 
 occ_status check_launch(const char* what) {
   cudaError_t e = cudaGetLastError();
@@ -52,6 +58,8 @@ const char* occ_status_string(occ_status s) {
 }
 
 const char* occ_last_error(void) { return occ::g_msg; }
+
+const char* occ_last_kernel(void) { return occ::g_kernel; }
 
 int occ_version(void) { return OCC_VERSION; }
 

@@ -284,6 +284,7 @@ extern "C" occ_status occ_ewma_update(float* theta_prox, const float* theta, int
   const int64_t blocks_cap = (int64_t)sm_count() * 8;
   if (aligned(theta_prox, 16) && aligned(theta, 16)) {
     const int64_t n4 = n / 4;
+    note_kernel(n4 > 0 ? "k3_ewma_vec" : "k3_ewma_scalar");
     if (n4 > 0) {
       const int64_t need = (n4 + kK3Threads * kK3Unroll - 1) / (kK3Threads * kK3Unroll);
       const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
@@ -293,6 +294,7 @@ extern "C" occ_status occ_ewma_update(float* theta_prox, const float* theta, int
     if (n - n4 * 4 > 0)
       k3_ewma_scalar<kK3Threads><<<1, kK3Threads, 0, s>>>(theta_prox, theta, n4 * 4, n, st);
   } else {
+    note_kernel("k3_ewma_scalar");
     const int64_t need = (n + kK3Threads - 1) / kK3Threads;
     const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
     k3_ewma_scalar<kK3Threads><<<grid, kK3Threads, 0, s>>>(theta_prox, theta, 0, n, st);
@@ -335,6 +337,7 @@ occ_status launch_bf16_body(bf16_t* tp, const void* th, occ_dtype theta_dt, int6
   auto grid_for = [&](int per_sm) {
     return (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, (int64_t)sm_count() * per_sm));
   };
+  note_kernel("k3_ewma_bf16");
   if (theta_dt == OCC_BF16)
     k3_ewma_bf16<bf16_t, kK3Threads, kK3Unroll>
         <<<grid_for(k3_bf16_ctas_per_sm<bf16_t>()), kK3Threads, 0, s>>>(tp, (const bf16_t*)th, n,
@@ -353,6 +356,7 @@ occ_status launch_f32_body(float* tp, const float* th, int64_t n, const occ_ewma
   const int64_t blocks_cap = (int64_t)sm_count() * 8;
   if (aligned(tp, 16) && aligned(th, 16)) {
     const int64_t n4 = n / 4;
+    note_kernel(n4 > 0 ? "k3_ewma_vec" : "k3_ewma_scalar");
     if (n4 > 0) {
       const int64_t need = (n4 + kK3Threads * kK3Unroll - 1) / (kK3Threads * kK3Unroll);
       const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
@@ -361,6 +365,7 @@ occ_status launch_f32_body(float* tp, const float* th, int64_t n, const occ_ewma
     }
     if (n - n4 * 4 > 0) k3_ewma_scalar<kK3Threads><<<1, kK3Threads, 0, s>>>(tp, th, n4 * 4, n, st);
   } else {
+    note_kernel("k3_ewma_scalar");
     const int64_t need = (n + kK3Threads - 1) / kK3Threads;
     const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
     k3_ewma_scalar<kK3Threads><<<grid, kK3Threads, 0, s>>>(tp, th, 0, n, st);

@@ -19,7 +19,10 @@
 namespace occ {
 
 // Vector path: 16-byte rows.  U vectors of each row in flight per thread.
-template <typename Tin, typename Tout, int NT, int U, bool DIAG>
+// PEEL: rows that start off a 16-byte boundary take their first `lead`
+// elements (up to the boundary) as scalars; the old-logits and gradient rows
+// have the same byte offset (checked on the host).
+template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
@@ -30,29 +33,37 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
   const uint64_t last = l2_policy_evict_first();
   const int tid = threadIdx.x;
   const int64_t V = a.V;
-  const int64_t nvec = V / VEC;
-  const int64_t tail0 = nvec * VEC;
-  const int64_t head = min(nvec, (int64_t)(a.stage_bytes / 16));
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
   for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
     const int id = a.ids[row];
     const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
     const bool id_ok = id >= 0 && (int64_t)id < V;
-    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    const Tin* z0 = (const Tin*)a.logits + row * a.ld;
+    const Tin* zo0 = (const Tin*)f.logits_old + row * f.ld_old;
+    const int64_t lead =
+        PEEL ? min(V, (int64_t)(((16 - ((uintptr_t)z0 & 15)) & 15) / sizeof(Tin))) : 0;
+    const Tin* z = z0 + lead;
+    const Tin* zo = zo0 + lead;
+    const int64_t nvec = (V - lead) / VEC;
+    const int64_t tail0 = nvec * VEC;  // relative to z
+    const int64_t ntail = V - lead - tail0;
+    const int64_t head = min(nvec, (int64_t)(a.stage_bytes / 16));
+    const int idr = id - (int)lead;  // the sampled token relative to z
+    Tout* drow0 = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    Tout* drow = drow0 ? drow0 + lead : nullptr;
     if (!(m && id_ok)) {
       if (drow) {
         for (int64_t i = tid; i < nvec; i += NT) OutVecHint<Tout, VEC>::zero(drow + i * VEC, last);
-        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+        if ((int64_t)tid < ntail) out_scalar(drow + tail0 + tid, 0.f);
+        if (PEEL && (int64_t)tid < lead) out_scalar(drow0 + tid, 0.f);
       }
       if (tid == 0) fused_dropped_outputs(f, row, m, id_ok);
       continue;
     }
-    const Tin* z = (const Tin*)a.logits + row * a.ld;
-    const Tin* zo = (const Tin*)f.logits_old + row * f.ld_old;
     float zy = 0.f, zyo = 0.f, lpm = 0.f, A = 0.f;
     if (tid == 0) {
-      zy = Elem<Tin>::load(z + id);
-      zyo = Elem<Tin>::load(zo + id);
+      zy = Elem<Tin>::load(z0 + id);
+      zyo = Elem<Tin>::load(zo0 + id);
       lpm = a.lp_mu[row];
       A = a.adv[row];
     }
@@ -71,6 +82,11 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
       accv_add<VEC, DIAG>(acc[0], x, x);
       accv_add<VEC, DIAG>(acc[1], xo, d);
     };
+    auto consume1 = [&](float xs, float xos) {
+      float x1[1] = {xs}, xo1[1] = {xos}, d1[1] = {xos - xs};
+      accv_add<1, DIAG>(acc[0], x1, x1);
+      accv_add<1, DIAG>(acc[1], xo1, d1);
+    };
     int64_t i = tid;
     for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
       uint4 rt[U], ro[U];
@@ -83,13 +99,14 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
       for (int u = 0; u < U; ++u) consume(i + u * NT, rt[u], ro[u]);
     }
     for (; i < nvec; i += NT) consume(i, ld_hint_v4(zv + i, keep), ld_hint_v4(zov + i, last));
-    float xt = 0.f;
-    if ((int64_t)tid < V - tail0) {
+    float xt = 0.f, xp = 0.f;
+    if ((int64_t)tid < ntail) {
       xt = Elem<Tin>::load(z + tail0 + tid);
-      const float xot = Elem<Tin>::load(zo + tail0 + tid);
-      float x1[1] = {xt}, xo1[1] = {xot}, d1[1] = {xot - xt};
-      accv_add<1, DIAG>(acc[0], x1, x1);
-      accv_add<1, DIAG>(acc[1], xo1, d1);
+      consume1(xt, Elem<Tin>::load(zo + tail0 + tid));
+    }
+    if (PEEL && (int64_t)tid < lead) {
+      xp = Elem<Tin>::load(z0 + tid);
+      consume1(xp, Elem<Tin>::load(zo0 + tid));
     }
     float C[2], SV[2];
     float2 S[2];
@@ -105,7 +122,8 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
       const float g = bc_g, cb = bc_cb;
       if (g == 0.f) {
         for (int64_t j = tid; j < nvec; j += NT) OutVecHint<Tout, VEC>::zero(drow + j * VEC, last);
-        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+        if ((int64_t)tid < ntail) out_scalar(drow + tail0 + tid, 0.f);
+        if (PEEL && (int64_t)tid < lead) out_scalar(drow0 + tid, 0.f);
       } else {
         const float sgn = g > 0.f ? -1.f : 1.f;
         auto emit = [&](int64_t jj, const uint4& r) {
@@ -113,10 +131,10 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
           Elem<Tin>::unpack(r, x);
 #pragma unroll
           for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
-          if (id >= jj * VEC && id < (jj + 1) * VEC) {
+          if (idr >= jj * VEC && idr < (jj + 1) * VEC) {
 #pragma unroll
             for (int q = 0; q < VEC; ++q)
-              if (jj * VEC + q == id) d[q] += g;
+              if (jj * VEC + q == idr) d[q] += g;
           }
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
@@ -132,10 +150,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
         for (; k < nre; k += NT) emit(head + k, ld_hint_v4(zv + (head + k), last));
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
-        if ((int64_t)tid < V - tail0) {
+        if ((int64_t)tid < ntail) {
           float dv = sgn * ex2_approx(fmaf(xt, kLog2e, -cb));
-          if (tail0 + tid == id) dv += g;
+          if (tail0 + tid == idr) dv += g;
           out_scalar(drow + tail0 + tid, dv);
+        }
+        if (PEEL && (int64_t)tid < lead) {
+          float dv = sgn * ex2_approx(fmaf(xp, kLog2e, -cb));
+          if (tid == id) dv += g;
+          out_scalar(drow0 + tid, dv);
         }
       }
     }
@@ -232,13 +255,41 @@ static bool fused_ring_selected() {
 template <typename Tin, typename Tout>
 occ_status launch_fused_ring(const FusedArgs& f, cudaStream_t s);
 
+using FusedKern = void (*)(const FusedArgs);
+
+template <typename Tin, typename Tout, bool DIAG, bool PEEL>
+static FusedKern fused_kernel(int nt) {
+  return nt == 128   ? k2_fused_l2<Tin, Tout, 128, kFusedUnroll, DIAG, PEEL>
+         : nt == 256 ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, DIAG, PEEL>
+                     : k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, DIAG, PEEL>;
+}
+
+// Rows off a 16-byte boundary run the vector kernel peeled when the old-logits
+// and gradient rows sit at the same byte offsets as the current-logits rows
+// (same element size; base addresses and row strides congruent modulo 16
+// bytes) and a row holds at least a few vectors.
+template <typename Tin, typename Tout>
+static bool fused_peel_ok(const FusedArgs& f) {
+  const K2Args& a = f.a;
+  const int64_t es = (int64_t)sizeof(Tin);
+  if (sizeof(Tout) != sizeof(Tin)) return false;
+  if (a.V < 16 * Elem<Tin>::kVec || ((uintptr_t)a.logits % es) != 0) return false;
+  if ((((uintptr_t)f.logits_old - (uintptr_t)a.logits) % 16) != 0 ||
+      (((f.ld_old - a.ld) * es) % 16) != 0)
+    return false;
+  if (!a.dlogits) return true;
+  return (((uintptr_t)a.dlogits - (uintptr_t)a.logits) % 16) == 0 &&
+         (((a.ld_grad - a.ld) * es) % 16) == 0;
+}
+
 template <typename Tin, typename Tout, bool DIAG>
 static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
   const int64_t T = f.a.T;
   const int64_t step = 0x7fffffffLL;
   if (vec && !DIAG && f.a.V >= Elem<Tin>::kVec && fused_ring_selected())
     return launch_fused_ring<Tin, Tout>(f, s);
-  if (vec) {
+  const bool peel = !vec && fused_peel_ok<Tin, Tout>(f);
+  if (vec || peel) {
     static const int nt_env = [] {
       const char* e = getenv("OCC_FUSED_THREADS");
       return e ? atoi(e) : 0;
@@ -257,9 +308,9 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
     const size_t head_auto = nt_auto == kFusedThreads ? kFusedHeadBytes : 0;
     const size_t head = std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
     f.a.stage_bytes = (int64_t)head;
-    auto kern = nt == 128   ? k2_fused_l2<Tin, Tout, 128, kFusedUnroll, DIAG>
-                : nt == 256 ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, DIAG>
-                            : k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, DIAG>;
+    FusedKern kern = fused_kernel<Tin, Tout, DIAG, false>(nt);
+    if constexpr (sizeof(Tin) == sizeof(Tout))
+      if (peel) kern = fused_kernel<Tin, Tout, DIAG, true>(nt);
     if (head > 0) {
       cudaError_t e =
           cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)head);
@@ -267,11 +318,13 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
         return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head,
                     cudaGetErrorString(e));
     }
+    note_kernel(peel ? "k2_fused_l2/peel" : "k2_fused_l2");
     for (int64_t r0 = 0; r0 < T; r0 += step) {
       f.a.row0 = r0;
       kern<<<(unsigned)std::min<int64_t>(step, T - r0), nt, head, s>>>(f);
     }
   } else {
+    note_kernel("k2_fused_stream");
     for (int64_t r0 = 0; r0 < T; r0 += step) {
       f.a.row0 = r0;
       k2_fused_stream<Tin, Tout, kFusedThreads, DIAG>

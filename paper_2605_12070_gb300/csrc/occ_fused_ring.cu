@@ -407,6 +407,7 @@ static occ_status launch_fused_ring_geo(const FusedArgs& f, cudaStream_t s) {
     return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", Gm::kSmem,
                 cudaGetErrorString(e));
   const unsigned grid = (unsigned)std::min<int64_t>(f.a.T, sm_count());
+  note_kernel("k2_fused_ring");
   kern<<<grid, Gm::kNT, Gm::kSmem, s>>>(f);
   return check_launch("occ_decoupled_loss_fused (ring)");
 }

@@ -10,8 +10,10 @@ namespace occ {
 
 // Records a printf-style message for occ_last_error() and returns `s`.
 occ_status fail(occ_status s, const char* fmt, ...);
-// Clears the message of the calling thread.
+// Clears the message and the launched-kernel name of the calling thread.
 void clear_error();
+// Records `name` (a string literal) for occ_last_kernel().
+void note_kernel(const char* name);
 // Maps a CUDA error (after a launch) to OCC_ERR_CUDA with a message.
 occ_status check_launch(const char* what);
 

@@ -15,22 +15,28 @@ namespace occ {
 constexpr int kK1Threads = 512;
 constexpr int kK1Unroll = 8;
 
-template <typename Tin, int NT, int U>
+// PEEL: rows need not start on a 16-byte boundary.  Each row then takes its
+// first `lead` elements (up to the boundary) and its last few with scalar
+// loads and the aligned body with the vector loop.
+template <typename Tin, int NT, int U, bool PEEL>
 __global__ void __launch_bounds__(NT, 1024 / NT)
     k1_logprob_vec(const Tin* __restrict__ logits, int64_t T, int64_t V, int64_t ld,
                    const int32_t* __restrict__ ids, float* __restrict__ logp,
                    float* __restrict__ lse_out) {
   constexpr int VEC = Elem<Tin>::kVec;
   __shared__ RedScratch red;
-  const int64_t nvec = V / VEC;
-  const int64_t tail0 = nvec * VEC;
   for (int64_t row = blockIdx.x; row < T; row += gridDim.x) {
-    const Tin* z = logits + row * ld;
+    const Tin* z0 = logits + row * ld;
+    const int64_t lead =
+        PEEL ? min(V, (int64_t)(((16 - ((uintptr_t)z0 & 15)) & 15) / sizeof(Tin))) : 0;
+    const Tin* z = z0 + lead;  // 16-byte aligned
+    const int64_t nvec = (V - lead) / VEC;
+    const int64_t tail0 = nvec * VEC;  // relative to z
     int id = 0;
     float zy = 0.f;
     if (threadIdx.x == 0) {
       id = ids[row];
-      if (id >= 0 && id < V) zy = Elem<Tin>::load(z + id);
+      if (id >= 0 && id < V) zy = Elem<Tin>::load(z0 + id);
     }
     LseAcc acc;
     acc_init(acc);
@@ -52,8 +58,12 @@ __global__ void __launch_bounds__(NT, 1024 / NT)
       Elem<Tin>::unpack(ld_stream_v4(zv + i), x);
       acc_add(acc, x);
     }
-    if ((int64_t)threadIdx.x < V - tail0) {
+    if ((int64_t)threadIdx.x < V - lead - tail0) {
       float x[1] = {Elem<Tin>::load(z + tail0 + threadIdx.x)};
+      acc_add(acc, x);
+    }
+    if (PEEL && (int64_t)threadIdx.x < lead) {
+      float x[1] = {Elem<Tin>::load(z0 + threadIdx.x)};
       acc_add(acc, x);
     }
     float C;
@@ -114,23 +124,29 @@ static void launch_k1(const void* logits, int64_t T, int64_t V, int64_t ld, cons
     const char* e = getenv("OCC_K1_THREADS");
     return e ? atoi(e) : 0;
   }();
-  if (vec) {
+  if (vec || V >= 16 * Elem<Tin>::kVec) {
     // rows up to ~96 KB: 128 threads; longer rows: 256 (measured on GB300 from
-    // V = 32000 to 151936 bf16; 512 threads left 2-50 % on the table)
+    // V = 32000 to 151936 bf16; 512 threads left 2-50 % on the table).  Rows
+    // that are not 16-byte aligned run peeled (scalar head and tail).
     const int64_t row_bytes = (V / Elem<Tin>::kVec) * 16;
     const int nt = nt_env ? nt_env : (row_bytes <= 96 * 1024 ? 128 : 256);
-    if (nt == 128)
-      k1_logprob_vec<Tin, 128, kK1Unroll><<<grid, 128, 0, s>>>((const Tin*)logits, T, V, ld, ids,
-                                                              logp, lse);
-    else if (nt == 256)
-      k1_logprob_vec<Tin, 256, kK1Unroll><<<grid, 256, 0, s>>>((const Tin*)logits, T, V, ld, ids,
-                                                              logp, lse);
-    else
-      k1_logprob_vec<Tin, kK1Threads, kK1Unroll><<<grid, kK1Threads, 0, s>>>(
-          (const Tin*)logits, T, V, ld, ids, logp, lse);
-  } else
+    const Tin* z = (const Tin*)logits;
+#define OCC_K1_LAUNCH(NT_, PEEL_) \
+  k1_logprob_vec<Tin, NT_, kK1Unroll, PEEL_><<<grid, NT_, 0, s>>>(z, T, V, ld, ids, logp, lse)
+    note_kernel(vec ? "k1_logprob_vec" : "k1_logprob_vec/peel");
+    if (nt == 128) {
+      if (vec) OCC_K1_LAUNCH(128, false); else OCC_K1_LAUNCH(128, true);
+    } else if (nt == 256) {
+      if (vec) OCC_K1_LAUNCH(256, false); else OCC_K1_LAUNCH(256, true);
+    } else {
+      if (vec) OCC_K1_LAUNCH(kK1Threads, false); else OCC_K1_LAUNCH(kK1Threads, true);
+    }
+#undef OCC_K1_LAUNCH
+  } else {
+    note_kernel("k1_logprob_scalar");
     k1_logprob_scalar<Tin, kK1Threads><<<grid, kK1Threads, 0, s>>>((const Tin*)logits, T, V, ld,
                                                                     ids, logp, lse);
+  }
 }
 
 }  // namespace occ

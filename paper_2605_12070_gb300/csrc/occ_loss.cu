@@ -561,7 +561,7 @@ __global__ void __launch_bounds__(NT, 2) k2_loss_reg(const K2Args a) {
 // sees the logits once and dlogits once.  Oldest-first bounds the time a line
 // waits in L2 by the longer of the two passes (newest-first lets the first
 // lines wait through both).  dlogits are written evict-first.
-template <typename Tin, typename Tout, int NT, int U>
+template <typename Tin, typename Tout, int NT, int U, bool PEEL>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
@@ -571,27 +571,36 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   const uint64_t last = l2_policy_evict_first();
   const int tid = threadIdx.x;
   const int64_t V = a.V;
-  const int64_t nvec = V / VEC;
-  const int64_t tail0 = nvec * VEC;
-  const int64_t head = min(nvec, (int64_t)(a.stage_bytes / 16));  // vectors kept on chip
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
   for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
     const int id = a.ids[row];
     const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
     const bool id_ok = id >= 0 && (int64_t)id < V;
-    Tout* drow = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    // PEEL: the row's first `lead` elements (up to its 16-byte boundary) are
+    // scalar; the gradient row has the same byte offset (checked on the host)
+    const Tin* z0 = (const Tin*)a.logits + row * a.ld;
+    const int64_t lead =
+        PEEL ? min(V, (int64_t)(((16 - ((uintptr_t)z0 & 15)) & 15) / sizeof(Tin))) : 0;
+    const Tin* z = z0 + lead;
+    const int64_t nvec = (V - lead) / VEC;
+    const int64_t tail0 = nvec * VEC;  // relative to z
+    const int64_t ntail = V - lead - tail0;
+    const int64_t head = min(nvec, (int64_t)(a.stage_bytes / 16));  // vectors kept on chip
+    const int idr = id - (int)lead;  // the sampled token relative to z
+    Tout* drow0 = a.dlogits ? (Tout*)a.dlogits + row * a.ld_grad : nullptr;
+    Tout* drow = drow0 ? drow0 + lead : nullptr;
     if (!(m && id_ok)) {
       if (drow) {
         for (int64_t i = tid; i < nvec; i += NT) OutVecHint<Tout, VEC>::zero(drow + i * VEC, last);
-        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+        if ((int64_t)tid < ntail) out_scalar(drow + tail0 + tid, 0.f);
+        if (PEEL && (int64_t)tid < lead) out_scalar(drow0 + tid, 0.f);
       }
       if (tid == 0) dropped_token_outputs(a, row, m, id_ok);
       continue;
     }
-    const Tin* z = (const Tin*)a.logits + row * a.ld;
     float zy = 0.f, lpo = 0.f, lpm = 0.f, A = 0.f;
     if (tid == 0) {
-      zy = Elem<Tin>::load(z + id);
+      zy = Elem<Tin>::load(z0 + id);
       lpo = a.lp_old ? a.lp_old[row] : 0.f;
       lpm = a.lp_mu[row];
       A = a.adv[row];
@@ -620,10 +629,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
       Elem<Tin>::unpack(r, x);
       acc_add_fast(acc, x);
     }
-    float xt = 0.f;
-    if ((int64_t)tid < V - tail0) {
+    float xt = 0.f, xp = 0.f;
+    if ((int64_t)tid < ntail) {
       xt = Elem<Tin>::load(z + tail0 + tid);
       float x1[1] = {xt};
+      acc_add(acc, x1);
+    }
+    if (PEEL && (int64_t)tid < lead) {
+      xp = Elem<Tin>::load(z0 + tid);
+      float x1[1] = {xp};
       acc_add(acc, x1);
     }
     float Cr;
@@ -652,7 +666,8 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
       const float g = bc_g, cb = bc_cb;
       if (g == 0.f) {
         for (int64_t j = tid; j < nvec; j += NT) OutVecHint<Tout, VEC>::zero(drow + j * VEC, last);
-        if ((int64_t)tid < V - tail0) out_scalar(drow + tail0 + tid, 0.f);
+        if ((int64_t)tid < ntail) out_scalar(drow + tail0 + tid, 0.f);
+        if (PEEL && (int64_t)tid < lead) out_scalar(drow0 + tid, 0.f);
       } else {
         const float sgn = g > 0.f ? -1.f : 1.f;
         auto emit = [&](int64_t jj, const uint4& r) {
@@ -660,10 +675,10 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
           Elem<Tin>::unpack(r, x);
 #pragma unroll
           for (int q = 0; q < VEC; ++q) d[q] = sgn * ex2_approx(fmaf(x[q], kLog2e, -cb));
-          if (id >= jj * VEC && id < (jj + 1) * VEC) {
+          if (idr >= jj * VEC && idr < (jj + 1) * VEC) {
 #pragma unroll
             for (int q = 0; q < VEC; ++q)
-              if (jj * VEC + q == id) d[q] += g;
+              if (jj * VEC + q == idr) d[q] += g;
           }
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
@@ -681,10 +696,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
         // on-chip head
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
-        if ((int64_t)tid < V - tail0) {
+        if ((int64_t)tid < ntail) {
           float dv = sgn * ex2_approx(fmaf(xt, kLog2e, -cb));
-          if (tail0 + tid == id) dv += g;
+          if (tail0 + tid == idr) dv += g;
           out_scalar(drow + tail0 + tid, dv);
+        }
+        if (PEEL && (int64_t)tid < lead) {
+          float dv = sgn * ex2_approx(fmaf(xp, kLog2e, -cb));
+          if (tid == id) dv += g;
+          out_scalar(drow0 + tid, dv);
         }
       }
     }
@@ -895,14 +915,41 @@ static int k2_variant() {
   return v;
 }
 
+using K2Kern = void (*)(const K2Args);
+
+template <typename Tin, typename Tout, bool PEEL>
+static K2Kern l2_kernel(int var, int nt, int unroll) {
+  return (var == 3)      ? k2_loss_l2<Tin, Tout, 1024, 8, PEEL>
+         : (nt == 128)   ? k2_loss_l2<Tin, Tout, 128, 8, PEEL>
+         : (nt == 256)   ? k2_loss_l2<Tin, Tout, 256, 8, PEEL>
+         : (unroll == 4) ? k2_loss_l2<Tin, Tout, 512, 4, PEEL>
+                         : k2_loss_l2<Tin, Tout, 512, 8, PEEL>;
+}
+
+// Rows that are not 16-byte aligned can run the vector kernel peeled when the
+// gradient rows sit at the same byte offsets as the logits rows (same element
+// size, base addresses and row strides congruent modulo 16 bytes) and a row
+// holds at least a few vectors.  Only the same-size instantiations exist.
+template <typename Tin, typename Tout>
+static bool k2_peel_ok(const K2Args& a) {
+  const int64_t es = (int64_t)sizeof(Tin);
+  if (sizeof(Tout) != sizeof(Tin)) return false;
+  if (a.V < 16 * Elem<Tin>::kVec || ((uintptr_t)a.logits % es) != 0) return false;
+  if (!a.dlogits) return true;
+  return (((uintptr_t)a.dlogits - (uintptr_t)a.logits) % 16) == 0 &&
+         (((a.ld_grad - a.ld) * es) % 16) == 0;
+}
+
 template <typename Tin, typename Tout>
 static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
   const int64_t T = a.T;
-  if (vec) {
-    const int var = k2_variant();
+  const bool peel = !vec && k2_peel_ok<Tin, Tout>(a);
+  if (vec || peel) {
+    const int var = vec ? k2_variant() : 0;  // the cluster variants need aligned rows
     if (var == 1) {
       const ClusterPlan pr = plan_reg(a.V, sizeof(Tin), kK2Stages);
       if (pr.C > 0) {
+        note_kernel("k2_loss_reg");
         constexpr int EV = (int)(kRegSliceElems / kRegThreads / Elem<Tin>::kVec);
         return launch_persistent(k2_loss_reg<Tin, Tout, kRegThreads, EV, kK2Stages>, kRegThreads,
                                  a, pr, kK2Stages, s);
@@ -911,6 +958,7 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     if (var == 2) {
       const ClusterPlan pl = plan_cluster(a.V, sizeof(Tin), kK2Stages);
       if (pl.C > 0) {
+        note_kernel("k2_loss_tma");
         if (k2_threads() == 512)
           return launch_persistent(k2_loss_tma<Tin, Tout, 512, kK2Stages>, 512, a, pl, kK2Stages,
                                    s);
@@ -940,11 +988,9 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
       return e ? atoi(e) : 0;
     }();
     const int nt_small = nt_env ? nt_env : nt_auto;
-    auto kern = (var == 3)            ? k2_loss_l2<Tin, Tout, 1024, 8>
-                : (nt_small == 128) ? k2_loss_l2<Tin, Tout, 128, 8>
-                : (nt_small == 256) ? k2_loss_l2<Tin, Tout, 256, 8>
-                : (unroll == 4)       ? k2_loss_l2<Tin, Tout, 512, 4>
-                                      : k2_loss_l2<Tin, Tout, 512, 8>;
+    K2Kern kern = l2_kernel<Tin, Tout, false>(var, nt_small, unroll);
+    if constexpr (sizeof(Tin) == sizeof(Tout))
+      if (peel) kern = l2_kernel<Tin, Tout, true>(var, nt_small, unroll);
     const int nt = (var == 3) ? 1024 : (nt_small == 128 || nt_small == 256) ? nt_small : 512;
     if (head_bytes > 0) {
       cudaError_t e =
@@ -953,6 +999,7 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
         return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head_bytes,
                     cudaGetErrorString(e));
     }
+    note_kernel(peel ? "k2_loss_l2/peel" : "k2_loss_l2");
     const int64_t step = 0x7fffffffLL;
     for (int64_t r0 = 0; r0 < T; r0 += step) {
       a.row0 = r0;
@@ -961,6 +1008,7 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     }
     return check_launch("occ_decoupled_loss_fwd_bwd");
   }
+  note_kernel("k2_loss_stream");
   const int64_t step = 0x7fffffffLL;
   for (int64_t r0 = 0; r0 < T; r0 += step) {
     a.row0 = r0;

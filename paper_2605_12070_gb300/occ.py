@@ -37,7 +37,7 @@ EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_
            "occ_decoupled_loss_fused", "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update",
            "occ_ewma_update_bf16", "occ_ewma_update_host", "occ_ewma_state_init",
            "occ_host_alloc", "occ_host_free", "occ_status_string", "occ_last_error",
-           "occ_version")
+           "occ_last_kernel", "occ_version")
 
 
 class OccError(RuntimeError):
@@ -112,10 +112,17 @@ def lib():
     L.occ_status_string.restype = ctypes.c_char_p
     L.occ_last_error.argtypes = []
     L.occ_last_error.restype = ctypes.c_char_p
+    L.occ_last_kernel.argtypes = []
+    L.occ_last_kernel.restype = ctypes.c_char_p
     L.occ_version.argtypes = []
     L.occ_version.restype = ctypes.c_int
     _lib = L
     return L
+
+
+def occ_last_kernel():
+    """The row kernel that the last occ call on this thread launched ("" if none)."""
+    return lib().occ_last_kernel().decode()
 
 
 def _check(rc, what):

@@ -137,7 +137,37 @@ def test_fused_strided_and_misaligned(layout):
                   (torch.rand(T, generator=g, device="cuda") < 0.8).to(torch.uint8),
                   rd_lo=0.7, rd_hi=1.4)
     out = _fused(b, want_diagnostics=True)
+    assert occ.occ_last_kernel() == "k2_fused_stream"  # rows at different byte offsets
     _check_fused(b, out, rows_dz=np.arange(T))
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("diag", [True, False])
+def test_fused_misaligned_rows_with_matching_layouts(dtype, diag):
+    """Current, old and gradient rows all one element past a 16-byte boundary
+    with one odd stride: the peeled vector kernel, every row-start residue,
+    the sampled token in row 0's scalar prefix and in the last row's tail."""
+    g = torch.Generator(device="cuda").manual_seed(13)
+    T, V, off = 23, 3001, 1
+    ld = V + 2
+    bz, bo = (torch.empty((T, ld), dtype=dtype, device="cuda") for _ in range(2))
+    bd = torch.full((T, ld), 7.0, dtype=dtype, device="cuda")
+    z, zo, dz = bz[:, off:off + V], bo[:, off:off + V], bd[:, off:off + V]
+    z.copy_((torch.randn((T, V), generator=g, device="cuda") * 2).to(dtype))
+    zo.copy_((z.float() + 0.3 * torch.randn((T, V), generator=g, device="cuda")).to(dtype))
+    ids = torch.randint(0, V, (T,), generator=g, device="cuda", dtype=torch.int32)
+    ids[0], ids[-1] = 0, V - 1
+    lo64, _ = logprob_rows(zo, ids, np.arange(T))
+    lmu = torch.from_numpy(fp32(lo64 + np.random.default_rng(13).normal(0, 0.2, T))).cuda()
+    b = LossBatch("edge", z, zo, ids, lmu, torch.randn(T, generator=g, device="cuda"),
+                  (torch.rand(T, generator=g, device="cuda") < 0.8).to(torch.uint8),
+                  rd_lo=0.7, rd_hi=1.4)
+    b.mask[0] = b.mask[-1] = 1
+    out = _fused(b, dlogits=dz, want_diagnostics=diag)
+    assert occ.occ_last_kernel() == "k2_fused_l2/peel"
+    out["dlogits"] = dz
+    _check_fused(b, out, rows_dz=np.arange(T), diag=diag)
+    assert torch.all(bd[:, :off] == 7.0) and torch.all(bd[:, off + V:] == 7.0)
 
 
 def test_fused_in_place_bad_ids_and_empty():

@@ -61,9 +61,26 @@ def test_strided_and_misaligned_rows(dtype):
     g = torch.Generator(device="cuda").manual_seed(7)
     big = (torch.randn((9, 5000), generator=g, device="cuda") * 2).to(dtype)
     ids = torch.randint(0, 4097, (9,), generator=g, device="cuda", dtype=torch.int32)
-    _check(big[:, :4097], ids)        # ld = 5000 > V (vector path when aligned)
-    _check(big[:, 1:4098], ids)       # base offset by one element: scalar path
-    _check(big.reshape(-1)[: 9 * 4097].view(9, 4097), ids)  # ld = V = 4097: scalar path
+    _check(big[:, :4097], ids)        # ld = 5000 > V: aligned rows
+    assert occ.occ_last_kernel() == "k1_logprob_vec"
+    _check(big[:, 1:4098], ids)       # base offset by one element: peeled rows
+    assert occ.occ_last_kernel() == "k1_logprob_vec/peel"
+    _check(big.reshape(-1)[: 9 * 4097].view(9, 4097), ids)  # ld = V = 4097: peeled rows
+    assert occ.occ_last_kernel() == "k1_logprob_vec/peel"
+    _check(big[:, 1:51], ids % 50)    # too short to peel: element loads
+    assert occ.occ_last_kernel() == "k1_logprob_scalar"
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("V", [4097, 20003])
+def test_misaligned_rows_take_the_peeled_vector_kernel(dtype, V):
+    g = torch.Generator(device="cuda").manual_seed(V)
+    big = (torch.randn((17, V + 2), generator=g, device="cuda") * 2).to(dtype)
+    z = big[:, 1:V + 1]                    # odd stride, every row-start residue
+    ids = torch.randint(0, V, (17,), generator=g, device="cuda", dtype=torch.int32)
+    ids[0], ids[-1] = 0, V - 1             # row 0's scalar prefix, the last row's tail
+    _check(z, ids)
+    assert occ.occ_last_kernel() == "k1_logprob_vec/peel"
 
 
 def test_bad_ids_give_nan_and_empty():

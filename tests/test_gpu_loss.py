@@ -248,9 +248,47 @@ def test_strided_and_misaligned(dtype, layout):
     # dlogits into a padded buffer of its own stride
     dz_buf = torch.full((T, V + 7), 7.0, dtype=dtype, device="cuda")
     out = _run(b, fp32(lp_old64), dz=dz_buf[:, :V])
+    # gradient rows at other byte offsets than the logits rows: element loads
+    assert occ.occ_last_kernel() == ("k2_loss_l2" if layout == "ld_pad" else "k2_loss_stream")
     out["dlogits"] = dz_buf[:, :V]
     _compare(b, out, o, lp_th64, dz_rows=np.arange(T), lse=lse, out_f32=dtype == torch.float32)
     assert torch.all(dz_buf[:, V:] == 7.0)   # padding untouched
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("V", [3001, 20003])
+def test_misaligned_rows_with_matching_gradient_layout(dtype, V):
+    """Rows off a 16-byte boundary whose gradient rows have the same byte
+    offsets (a buffer of the same stride and offset, in place, or no gradient)
+    run the peeled vector kernel.  The odd row stride gives every row-start
+    residue; the sampled token of row 0 lies in its scalar prefix and that of
+    the last row in its scalar tail."""
+    T, off = 29, 1
+    b, lp_old64 = _edge_batch(T, V, dtype, seed=V + 1, ld=V + 1, offset=off)
+    stride = b.z_theta.stride(0)
+    assert stride % 2 == 1 and b.z_theta.data_ptr() % 16 != 0
+    lp_th64, lse = logprob_rows(b.z_theta, b.ids, np.arange(T))
+    o = oracle_loss(b, lp_th64, fp32(lp_old64), loss_params(b))
+    dz_buf = torch.full((T, stride), 7.0, dtype=dtype, device="cuda")
+    dz = dz_buf[:, off:off + V]
+    out = _run(b, fp32(lp_old64), dz=dz)
+    assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    out["dlogits"] = dz
+    _compare(b, out, o, lp_th64, dz_rows=np.arange(T), lse=lse, out_f32=dtype == torch.float32)
+    assert torch.all(dz_buf[:, :off] == 7.0) and torch.all(dz_buf[:, off + V:] == 7.0)
+    # in place over a copy with the same layout: the same kernel, the same bits
+    buf2 = torch.empty((T, stride), dtype=dtype, device="cuda")
+    z2 = buf2[:, off:off + V]
+    z2.copy_(b.z_theta)
+    lp_old = torch.from_numpy(fp32(lp_old64)).to("cuda")
+    out2 = occ.occ_decoupled_loss_fwd_bwd(z2, b.ids, lp_old, b.logp_mu, b.adv, b.mask,
+                                          dlogits="inplace", **b.thresholds())
+    assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    # forward only
+    out3 = _run(b, fp32(lp_old64), dz=None)
+    assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    assert torch.equal(z2, dz) and torch.equal(out2["stats"], out["stats"])
+    assert torch.equal(out3["stats"], out["stats"]) and torch.equal(out3["logp"], out["logp"])
 
 
 @pytest.mark.parametrize("V", [600_000, 900_001])

@@ -50,8 +50,9 @@ def test_host_validation_without_gpu(L):
     # V = 0 is rejected before any CUDA call
     rc = L.occ_token_logprob(null, 0, 4, 0, 0, null, null, null, null)
     assert rc == 1 and b"V >= 1" in L.occ_last_error()
-    # T = 0 is a no-op
+    # T = 0 is a no-op and launches nothing
     assert L.occ_token_logprob(null, 1, 0, 10, 10, null, null, null, null) == 0
+    assert L.occ_last_kernel() == b""
     # bad dtype
     assert L.occ_token_logprob(null, 7, 1, 10, 10, null, null, null, null) == 2
     # inverted band
