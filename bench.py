@@ -59,6 +59,10 @@ def parse_args():
     ap.add_argument("--loss-path", default="fused", choices=["fused", "two-call"],
                     help="fused: one launch reads old and current logits (occ_decoupled_loss_fused); "
                          "two-call: occ_token_logprob then occ_decoupled_loss_fwd_bwd")
+    ap.add_argument("--write-traffic", nargs=4, metavar=("CSV", "T", "N_VALID", "N_PARAMS"),
+                    help="no GPU: turn an ncu CSV of dram__bytes_{read,write}.sum (a run of this "
+                         "script with T tokens, N_VALID of them valid, and N_PARAMS EWMA "
+                         "parameters) into profiles/traffic_per_unit.json")
     return ap.parse_args()
 
 
@@ -175,6 +179,60 @@ def ncu_traffic():
             if k in KERNEL_SOURCES and v.get("source_hash") == kernel_source_hash(k)}
 
 
+# kernel-name prefix in an ncu launch list -> KERNEL_SOURCES key
+_TRAFFIC_KERNELS = {"k1_logprob_vec": "k1_token_logprob", "k2_loss_l2": "k2_decoupled_loss_fwd_bwd",
+                    "k2_fused_l2": "k12_decoupled_loss_fused", "k3_ewma_vec": "k3_ewma_update"}
+
+
+def write_traffic(csv_path, T, n_valid, n_params, command):
+    """Averages each kernel's DRAM bytes over its captured launches and stores
+    them per unit (tokens, valid tokens, parameters) with the kernel's source
+    hash in profiles/traffic_per_unit.json."""
+    import csv
+    with open(csv_path) as f:
+        rows = list(csv.DictReader([ln for ln in f if ln.startswith('"')]))
+    acc = {}
+    for r in rows:
+        name = r["Kernel Name"].split("(")[0].replace("void ", "").strip()
+        key = next((k for p, k in _TRAFFIC_KERNELS.items() if name.startswith(p)), None)
+        metric = r["Metric Name"]
+        if key and metric in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+            scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9}[r.get("Metric Unit",
+                                                                              "byte")]
+            v = float(r["Metric Value"].replace(",", "")) * scale
+            acc.setdefault(key, {}).setdefault(metric, []).append(v)
+    kernels = {}
+    for key, d in acc.items():
+        rd = sum(d["dram__bytes_read.sum"]) / len(d["dram__bytes_read.sum"])
+        wr = sum(d["dram__bytes_write.sum"]) / len(d["dram__bytes_write.sum"])
+        if key == "k1_token_logprob":
+            e = {"read_per_token": rd / T, "write_per_token": wr / T}
+        elif key == "k3_ewma_update":
+            e = {"read_per_param": rd / n_params, "write_per_param": wr / n_params}
+        else:
+            e = {"read_per_valid_token": rd / n_valid, "write_per_token": wr / T}
+        e["launches"] = len(d["dram__bytes_read.sum"])
+        e["source_hash"] = kernel_source_hash(key)
+        kernels[key] = e
+    out = {
+        "what": (f"DRAM bytes per unit from one ncu capture (dram__bytes_read.sum, "
+                 f"dram__bytes_write.sum) of a run with T={T} tokens ({n_valid} valid) and "
+                 f"{n_params} EWMA parameters, averaged over the captured launches of each "
+                 f"kernel; bench.py scales them to its workload by the units processed (valid "
+                 f"tokens for the logits reads of the loss kernels, tokens for everything else, "
+                 f"parameters for the EWMA). Writes are slightly under-counted: a single launch "
+                 f"leaves up to ~60 MB of dirty lines in L2. Each entry is valid while its "
+                 f"kernel's code (comments and layout aside) hashes to source_hash."),
+        "command": command,
+        "kernels": kernels,
+    }
+    path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
+    with open(path, "w") as f:
+        json.dump(out, f, indent=1)
+        f.write("\n")
+    return out
+
+
 def traffic_bytes(tr, name, T, n_valid, n_params):
     """DRAM bytes of one launch, scaled from the per-unit capture."""
     k = tr.get(name)
@@ -283,8 +341,22 @@ def cpu_baseline(batch, n_params_full, seconds):
 
 # ----------------------------------------------------------------- main
 
+TRAFFIC_COMMAND = (
+    "python bench.py --tokens 4096 --ewma-n 400000000 --steps 2 --warmup 1 --no-e2e "
+    "--no-cpu-baseline --no-graph > plain_small.log && ncu --metrics dram__bytes_read.sum,"
+    "dram__bytes_write.sum,lts__t_sector_hit_rate.pct,gpu__time_duration.sum --clock-control none "
+    "-k regex:k[0-9]_ -c 40 --csv --log-file traffic_small.csv python bench.py --tokens 4096 "
+    "--ewma-n 400000000 --steps 2 --warmup 1 --no-e2e --no-cpu-baseline --no-graph; then "
+    "python bench.py --write-traffic traffic_small.csv 4096 <valid tokens> 400000000")
+
+
 def main():
     args = parse_args()
+    if args.write_traffic:
+        csv_path, T, n_valid, n_params = args.write_traffic
+        out = write_traffic(csv_path, int(T), int(n_valid), int(n_params), TRAFFIC_COMMAND)
+        print(json.dumps(out["kernels"], indent=1))
+        return
     import torch
     import torch.distributed as dist
 

@@ -259,6 +259,12 @@ __global__ void __launch_bounds__(NT, k3_bf16_ctas_per_sm<ThT>())
 
 using namespace occ;
 
+namespace {
+// Launches the float32 update of n parameters (vector body + scalar tail).
+occ_status launch_f32_body(float* tp, const float* th, int64_t n, const occ_ewma_state* st,
+                           cudaStream_t s);
+}  // namespace
+
 extern "C" occ_status occ_ewma_update(float* theta_prox, const float* theta, int64_t n,
                                       double beta, occ_ewma_state* st,
                                       const occ_loss_stats* stats, double tau, int32_t min_streak,
@@ -281,25 +287,7 @@ extern "C" occ_status occ_ewma_update(float* theta_prox, const float* theta, int
   k3_ewma_prologue<<<1, 1, 0, s>>>(st, stats, beta, tau, min_streak, force_reset ? 1 : 0);
   occ_status rc = check_launch("k3_ewma_prologue");
   if (rc != OCC_OK || n == 0) return rc;
-  const int64_t blocks_cap = (int64_t)sm_count() * 8;
-  if (aligned(theta_prox, 16) && aligned(theta, 16)) {
-    const int64_t n4 = n / 4;
-    note_kernel(n4 > 0 ? "k3_ewma_vec" : "k3_ewma_scalar");
-    if (n4 > 0) {
-      const int64_t need = (n4 + kK3Threads * kK3Unroll - 1) / (kK3Threads * kK3Unroll);
-      const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
-      k3_ewma_vec<kK3Threads, kK3Unroll><<<grid, kK3Threads, 0, s>>>(
-          (float4*)theta_prox, (const float4*)theta, n4, st);
-    }
-    if (n - n4 * 4 > 0)
-      k3_ewma_scalar<kK3Threads><<<1, kK3Threads, 0, s>>>(theta_prox, theta, n4 * 4, n, st);
-  } else {
-    note_kernel("k3_ewma_scalar");
-    const int64_t need = (n + kK3Threads - 1) / kK3Threads;
-    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min(need, blocks_cap));
-    k3_ewma_scalar<kK3Threads><<<grid, kK3Threads, 0, s>>>(theta_prox, theta, 0, n, st);
-  }
-  return check_launch("occ_ewma_update");
+  return launch_f32_body(theta_prox, theta, n, st, s);
 }
 
 extern "C" occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* stream) {
