@@ -34,6 +34,7 @@ METRIC = "correction-loss tokens/s fwd+bwd at V=151936; HBM GB/s vs peak"
 WORKLOAD = "agentic_bf16_v151936"
 EWMA_BETA = 0.99
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0   # HBM3e spec-sheet figure, for context next to the measured peak
 
 
 def parse_args():
@@ -529,6 +530,7 @@ def main():
         roof[name] = {
             "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
             "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+            "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
             "traffic": traffic_bytes(traffic, name, T, n_valid, args.ewma_n),
             "algorithmic_bytes": byts, "ms": round(sec * 1e3, 4),
         }
