@@ -62,8 +62,8 @@ def parse_args():
                          "two-call: occ_token_logprob then occ_decoupled_loss_fwd_bwd")
     ap.add_argument("--write-traffic", nargs=4, metavar=("CSV", "T", "N_VALID", "N_PARAMS"),
                     help="no GPU: turn an ncu CSV of dram__bytes_{read,write}.sum (a run of this "
-                         "script with T tokens, N_VALID of them valid, and N_PARAMS EWMA "
-                         "parameters) into profiles/traffic_per_unit.json")
+                         "script on --workload with T tokens, N_VALID of them valid, and N_PARAMS "
+                         "EWMA parameters) into profiles/traffic_per_unit.json")
     return ap.parse_args()
 
 
@@ -166,18 +166,22 @@ def kernel_source_hash(name):
     return h.hexdigest()[:16]
 
 
-def ncu_traffic():
+def ncu_traffic(workload, V):
     """Per-unit DRAM bytes from the committed ncu summary
     (profiles/traffic_per_unit.json) for the kernels whose sources have not
-    changed since the capture."""
+    changed since the capture, when the loss batch is the captured one (its
+    recipe and V: per-token bytes depend on both; the EWMA's per-parameter
+    bytes do not)."""
     path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
     try:
         with open(path) as f:
             d = json.load(f)
     except Exception:
         return {}
+    same_batch = d.get("workload") == workload and d.get("V") == V
     return {k: v for k, v in d.get("kernels", {}).items()
-            if k in KERNEL_SOURCES and v.get("source_hash") == kernel_source_hash(k)}
+            if k in KERNEL_SOURCES and v.get("source_hash") == kernel_source_hash(k)
+            and (same_batch or k == "k3_ewma_update")}
 
 
 # kernel-name prefix in an ncu launch list -> KERNEL_SOURCES key
@@ -185,7 +189,7 @@ _TRAFFIC_KERNELS = {"k1_logprob_vec": "k1_token_logprob", "k2_loss_l2": "k2_deco
                     "k2_fused_l2": "k12_decoupled_loss_fused", "k3_ewma_vec": "k3_ewma_update"}
 
 
-def write_traffic(csv_path, T, n_valid, n_params, command):
+def write_traffic(csv_path, workload, V, T, n_valid, n_params, command):
     """Averages each kernel's DRAM bytes over its captured launches and stores
     them per unit (tokens, valid tokens, parameters) with the kernel's source
     hash in profiles/traffic_per_unit.json."""
@@ -225,6 +229,8 @@ def write_traffic(csv_path, T, n_valid, n_params, command):
                  f"leaves up to ~60 MB of dirty lines in L2. Each entry is valid while its "
                  f"kernel's code (comments and layout aside) hashes to source_hash."),
         "command": command,
+        "workload": workload,
+        "V": V,
         "kernels": kernels,
     }
     path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
@@ -355,7 +361,9 @@ def main():
     args = parse_args()
     if args.write_traffic:
         csv_path, T, n_valid, n_params = args.write_traffic
-        out = write_traffic(csv_path, int(T), int(n_valid), int(n_params), TRAFFIC_COMMAND)
+        from paper_2605_12070_gb300.workloads import WORKLOADS
+        out = write_traffic(csv_path, args.workload, WORKLOADS[args.workload]["V"], int(T),
+                            int(n_valid), int(n_params), TRAFFIC_COMMAND)
         print(json.dumps(out["kernels"], indent=1))
         return
     import torch
@@ -501,7 +509,7 @@ def main():
                  "launches_per_replay": 5 if args.loss_path == "fused" else 6}
 
     peak, peak_kind = measured_peak()
-    traffic = ncu_traffic()
+    traffic = ncu_traffic(args.workload, V)
     es = batch.z_theta.element_size()
     bytes_k1 = T * V * es + T * 8
     bytes_k2 = n_valid * V * es + T * V * es + T * 37
