@@ -41,6 +41,24 @@ int sm_count() {
   return n;
 }
 
+size_t two_cta_smem_budget(const void* kern) {
+  constexpr size_t kPerCta = (164 - 1) * 1024 / 2;
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  int dev = 0, reserve = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&reserve, cudaDevAttrReservedSharedMemoryPerBlock, dev) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  const size_t fixed = ((fa.sharedSizeBytes + 127) & ~(size_t)127) + (size_t)reserve;
+  return fixed < kPerCta ? ((kPerCta - fixed) & ~(size_t)511) : 0;
+}
+
 }  // namespace occ
 
 extern "C" {

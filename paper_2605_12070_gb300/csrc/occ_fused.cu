@@ -238,7 +238,6 @@ __global__ void __launch_bounds__(NT) k2_fused_stream(const FusedArgs f) {
 
 constexpr int kFusedThreads = 512;
 constexpr int kFusedUnroll = 4;
-constexpr size_t kFusedHeadBytes = 80 * 1024;
 
 // OCC_FUSED_VARIANT=ring selects the persistent TMA-ring kernel for the vector
 // path without diagnostics.
@@ -301,16 +300,20 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
     // Row-size tiers (measured on GB300, V = 32000 to 151936 bf16): short rows
     // finish in about one load round per CTA, so small CTAs, more of them per
     // SM and no shared-memory head (L2 holds every row in flight) keep the
-    // memory system busy; long rows want 512 threads and the 80 KB head.
+    // memory system busy; long rows want 512 threads and the largest head
+    // with which two CTAs stay in the 164 KB carveout (79 KB for this kernel;
+    // at 80 KB it crossed into the 196 KB carveout: 8.38 ms against 8.31 at
+    // V = 151936).
     const size_t row_bytes = (size_t)(f.a.V / Elem<Tin>::kVec) * 16;
     const int nt_auto = row_bytes <= 64 * 1024 ? 128 : row_bytes <= 112 * 1024 ? 256 : kFusedThreads;
     const int nt = nt_env ? nt_env : nt_auto;
-    const size_t head_auto = nt_auto == kFusedThreads ? kFusedHeadBytes : 0;
-    const size_t head = std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
-    f.a.stage_bytes = (int64_t)head;
     FusedKern kern = fused_kernel<Tin, Tout, DIAG, false>(nt);
     if constexpr (sizeof(Tin) == sizeof(Tout))
       if (peel) kern = fused_kernel<Tin, Tout, DIAG, true>(nt);
+    const size_t head_auto =
+        nt_auto == kFusedThreads ? two_cta_smem_budget((const void*)kern) : 0;
+    const size_t head = std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
+    f.a.stage_bytes = (int64_t)head;
     if (head > 0) {
       cudaError_t e =
           cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)head);

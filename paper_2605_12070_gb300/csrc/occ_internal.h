@@ -30,4 +30,13 @@ inline size_t dtype_size(occ_dtype dt) { return dt == OCC_BF16 ? 2 : 4; }
 // Multiprocessor count of the current device (cached per device).
 int sm_count();
 
+// Dynamic shared memory with which two CTAs of `kern` stay in the 164 KB
+// shared-memory carveout of an SM.  Past it the driver takes the 196 KB
+// carveout and L1, which holds the loads in flight, shrinks from ~92 KB to
+// ~60 KB (the fused kernel: 8.31 ms against 8.38 ms at V = 151936).  Measured
+// on GB300 with byte steps: a CTA may take half of 163 KB, counting its static
+// shared memory rounded up to 128 bytes and the per-CTA system reservation;
+// the result is rounded down to 512 bytes for margin.  0 if a query fails.
+size_t two_cta_smem_budget(const void* kern);
+
 }  // namespace occ

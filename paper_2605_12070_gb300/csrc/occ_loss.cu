@@ -967,7 +967,8 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     }
     // Row-size tiers (measured on GB300, V = 32000 to 151936 bf16): 128 threads
     // and a 16 KB head up to 64 KB rows, 256 threads and no head up to 112 KB,
-    // 512 threads and an 80 KB head beyond.  OCC_K2_L2_THREADS and
+    // 512 threads beyond, with the largest head that keeps two CTAs in the
+    // 164 KB shared-memory carveout (80 KB for this kernel).  OCC_K2_L2_THREADS and
     // OCC_K2_HEAD_KB override (0 = pure L2 re-read).
     const size_t row_bytes = (size_t)(a.V / Elem<Tin>::kVec) * 16;
     const int nt_auto = row_bytes <= 64 * 1024 ? 128 : row_bytes <= 112 * 1024 ? 256 : 512;
@@ -975,10 +976,6 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
       const char* e = getenv("OCC_K2_HEAD_KB");
       return e ? atol(e) * 1024 : -1L;
     }();
-    const size_t head_auto = nt_auto == 128 ? 16 * 1024 : nt_auto == 256 ? 0 : 80 * 1024;
-    const size_t head_bytes =
-        std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
-    a.stage_bytes = (int64_t)head_bytes;
     static const int unroll = [] {
       const char* e = getenv("OCC_K2_UNROLL");
       return e ? atoi(e) : 8;
@@ -991,6 +988,12 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     K2Kern kern = l2_kernel<Tin, Tout, false>(var, nt_small, unroll);
     if constexpr (sizeof(Tin) == sizeof(Tout))
       if (peel) kern = l2_kernel<Tin, Tout, true>(var, nt_small, unroll);
+    const size_t head_auto = nt_auto == 128   ? 16 * 1024
+                             : nt_auto == 256 ? 0
+                                              : two_cta_smem_budget((const void*)kern);
+    const size_t head_bytes =
+        std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
+    a.stage_bytes = (int64_t)head_bytes;
     const int nt = (var == 3) ? 1024 : (nt_small == 128 || nt_small == 256) ? nt_small : 512;
     if (head_bytes > 0) {
       cudaError_t e =
