@@ -11,6 +11,7 @@ import pytest
 import torch
 
 import oracle as orc
+from kernel_choice import expected_kernel
 from oracle_runner import dlogits_rows, fp32, logprob_rows, loss_params, oracle_loss
 from oracle.rows import to_f64
 from paper_2605_12070_gb300 import occ
@@ -214,7 +215,7 @@ def test_fused_full_size_agentic_sampled():
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 20000, 50000, 65536 + 3])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 20000, 50000, 65536 + 3])
 def test_fused_vocab_edges(V, dtype):
     # rows shorter than one vector, one vector exactly, a ragged tail after the
     # vector body, rows in each CTA-size tier (40 / 80 / 100 / 200 KB) and rows
@@ -231,6 +232,7 @@ def test_fused_vocab_edges(V, dtype):
                   (torch.rand(T, generator=g, device="cuda") < 0.8).to(torch.uint8),
                   rd_lo=0.7, rd_hi=1.4)
     out = _fused(b, want_diagnostics=True)
+    assert occ.occ_last_kernel() == expected_kernel("fused", V, z.element_size())
     _check_fused(b, out, rows_dz=np.arange(T))
     if V == 1:  # a one-token vocabulary: log pi = 0, entropy 0, KL 0
         v = b.mask.cpu().numpy().astype(bool)

@@ -9,6 +9,7 @@ import numpy as np
 import pytest
 import torch
 
+from kernel_choice import expected_kernel
 from oracle_runner import logprob_rows
 from paper_2605_12070_gb300 import occ
 from paper_2605_12070_gb300.workloads import make_loss_batch
@@ -47,13 +48,15 @@ def test_workloads_reduced(name, T):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 31, 4095, 4097, 20000, 50000, 151936])
+@pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 31, 63, 65, 127, 129, 4095, 4097, 20000, 50000,
+                               151936])
 def test_vocab_edges(V, dtype):
     g = torch.Generator(device="cuda").manual_seed(V)
     T = 5
     z = (torch.randn((T, V), generator=g, device="cuda") * 3).to(dtype)
     ids = torch.tensor([0, V - 1, V // 2, 0, V - 1], dtype=torch.int32, device="cuda")
     _check(z, ids)
+    assert occ.occ_last_kernel() == expected_kernel("k1", V, z.element_size())
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])

@@ -13,6 +13,7 @@ import pytest
 import torch
 
 from oracle import FLAG_ACTIVE, FLAG_CLIPPED, FLAG_IN_BAND, FLAG_VALID
+from kernel_choice import expected_kernel
 from oracle_runner import dlogits_rows, fp32, logprob_rows, loss_params, oracle_loss
 from paper_2605_12070_gb300 import occ
 from paper_2605_12070_gb300.workloads import make_loss_batch
@@ -225,7 +226,7 @@ def _edge_batch(T, V, dtype, seed, mask_p=0.8, ld=None, offset=0):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 4097, 20000, 50000, 65536 + 3])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 20000, 50000, 65536 + 3])
 def test_vocab_edges(V, dtype):
     T = 37
     b, lp_old64 = _edge_batch(T, V, dtype, seed=V)
@@ -233,6 +234,7 @@ def test_vocab_edges(V, dtype):
     p = loss_params(b)
     o = oracle_loss(b, lp_th64, fp32(lp_old64), p)
     out = _run(b, fp32(lp_old64))
+    assert occ.occ_last_kernel() == expected_kernel("k2", V, b.z_theta.element_size())
     _compare(b, out, o, lp_th64, dz_rows=np.arange(T), lse=lse,
              out_f32=dtype == torch.float32)
 
