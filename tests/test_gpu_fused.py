@@ -214,6 +214,37 @@ def test_fused_full_size_agentic_sampled():
     assert np.abs(out["kl"].cpu().numpy()[rows][v] - K[v]).max() <= DIAG_TOL
 
 
+def test_fused_odd_vocab_past_2_31_logits_sampled():
+    """An odd vocabulary (ld = V = 50257: rows off 16-byte boundaries, the
+    peeled kernel) over more than 2^31 logits per tensor, so row offsets pass
+    4 GB; sampled rows (the first, the last, random ones) against the oracle,
+    dlogits included."""
+    b = make_loss_batch("grpo_bf16_v32000", T=45_000, V=50_257, seed=6, device="cuda")
+    T, V = b.T, b.V
+    assert T * V > 2 ** 31
+    out = _fused(b)
+    assert occ.occ_last_kernel() == "k2_fused_l2/peel"
+    mask = np.ones(T, np.uint8) if b.mask is None else b.mask.cpu().numpy()
+    rng = np.random.default_rng(6)
+    rows = np.unique(np.concatenate([rng.choice(T, 96, replace=False), [0, 1, T - 2, T - 1]]))
+    lo64, _ = logprob_rows(b.z_old, b.ids, rows)
+    lt64, lse = logprob_rows(b.z_theta, b.ids, rows)
+    o = orc.token_terms(lt64, lo64, b.logp_mu.cpu().numpy()[rows], b.adv.cpu().numpy()[rows],
+                        mask[rows], loss_params(b), N=int(mask.sum()))
+    fl = out["flags"].cpu().numpy()[rows]
+    near = np.minimum(o["dist_rd"], o["dist_rs"]) <= EXEMPT
+    assert not ((fl != o["flags"]) & ~near).any()
+    v = o["valid"]
+    assert np.abs(out["logp"].cpu().numpy()[rows][v] - lt64[v]).max() <= 1e-5
+    assert np.abs(out["logp_old"].cpu().numpy()[rows][v] - lo64[v]).max() <= 1e-5
+    keep = fl == o["flags"]
+    assert np.count_nonzero(o["g"][keep]) > 0
+    ref = dlogits_rows(b, rows[keep], lse[keep], o["g"][keep])
+    got = out["dlogits"][torch.as_tensor(rows[keep], device="cuda")].float().cpu().numpy()
+    g = np.abs(o["g"][keep])[:, None]
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 4e-6 * g + 1e-30)
+
+
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
 @pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 20000, 50000, 65536 + 3])
 def test_fused_vocab_edges(V, dtype):
