@@ -557,20 +557,8 @@ def main():
         "vs_baseline": None,
         "dtype": "f32",
         "data": "synthetic",
-        "config": {
-            "workload": (f"decoupled-loss step on the {args.workload} batch, T={T} tokens "
-                         f"({n_valid} valid), V={V} {str(batch.z_theta.dtype).replace('torch.', '')} "
-                         f"old and current logits (log pi_old, loss fwd + dlogits) chained with the "
-                         f"PPO-EWMA update of {args.ewma_n} fp32 parameters"),
-            "loss_path": args.loss_path,
-            "T": T, "V": V, "ewma_params": args.ewma_n,
-            "logits_dtype": str(batch.z_theta.dtype).replace("torch.", ""),
-            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-            "l2": (f"inputs larger than L2 ({2 * T * V * es / 1e9:.0f} GB logits, "
-                   f"{8 * args.ewma_n / 1e9:.0f} GB EWMA buffers): no flush"),
-            "rd_band": [batch.rd_lo, batch.rd_hi], "eps": [batch.eps_low, batch.eps_high],
-            "tau": args.tau, "rho": round(st_last.rho, 5), "ewma_resets_timed": resets,
-        },
+        "config": dict(workload_config(args, batch, n_valid, world), loss_path=args.loss_path,
+                       rho=round(st_last.rho, 5), ewma_resets_timed=resets),
         "roofline": dict(roof[dominant], kernel=dominant),
         "kernels": roof,
         "loss_only": {"path": args.loss_path, "tokens_per_s": round(world * T / (k1 + k2), 1),
@@ -747,6 +735,25 @@ def run_ewma_variants(args, dev):
     print(json.dumps(out), flush=True)
 
 
+def workload_config(args, batch, n_valid, world):
+    """The workload part of the JSON line's config, shared by both arms."""
+    T, V = batch.T, batch.V
+    dt = str(batch.z_theta.dtype).replace("torch.", "")
+    es = batch.z_theta.element_size()
+    return {
+        "workload": (f"decoupled-loss step on the {args.workload} batch, T={T} tokens "
+                     f"({n_valid} valid), V={V} {dt} old and current logits (log pi_old, loss "
+                     f"fwd + dlogits) chained with the PPO-EWMA update of {args.ewma_n} fp32 "
+                     f"parameters"),
+        "T": T, "V": V, "ewma_params": args.ewma_n, "logits_dtype": dt,
+        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        "l2": (f"inputs larger than L2 ({2 * T * V * es / 1e9:.0f} GB logits, "
+               f"{8 * args.ewma_n / 1e9:.0f} GB EWMA buffers): no flush"),
+        "rd_band": [batch.rd_lo, batch.rd_hi], "eps": [batch.eps_low, batch.eps_high],
+        "tau": args.tau,
+    }
+
+
 def run_reference(args, batch, world):
     """The oracle as the reference arm: each step times the float64 oracle on a
     bounded sample of the same workload (host cores)."""
@@ -774,8 +781,7 @@ def run_reference(args, batch, world):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(step_s * 1e3, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": f"oracle on the same T={batch.T}, V={batch.V} step + "
-                               f"{args.ewma_n}-parameter EWMA update", "T": batch.T, "V": batch.V},
+        "config": dict(workload_config(args, batch, valid.size, world), loss_path="oracle"),
         "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": threads,
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
