@@ -166,13 +166,15 @@ def kernel_source_hash(name):
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload, V):
+TRAFFIC_JSON = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
+
+
+def ncu_traffic(workload, V, path=TRAFFIC_JSON):
     """Per-unit DRAM bytes from the committed ncu summary
     (profiles/traffic_per_unit.json) for the kernels whose sources have not
     changed since the capture, when the loss batch is the captured one (its
     recipe and V: per-token bytes depend on both; the EWMA's per-parameter
     bytes do not)."""
-    path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
     try:
         with open(path) as f:
             d = json.load(f)
@@ -189,7 +191,7 @@ _TRAFFIC_KERNELS = {"k1_logprob_vec": "k1_token_logprob", "k2_loss_l2": "k2_deco
                     "k2_fused_l2": "k12_decoupled_loss_fused", "k3_ewma_vec": "k3_ewma_update"}
 
 
-def write_traffic(csv_path, workload, V, T, n_valid, n_params, command):
+def write_traffic(csv_path, workload, V, T, n_valid, n_params, command, path=TRAFFIC_JSON):
     """Averages each kernel's DRAM bytes over its captured launches and stores
     them per unit (tokens, valid tokens, parameters) with the kernel's source
     hash in profiles/traffic_per_unit.json."""
@@ -233,7 +235,6 @@ def write_traffic(csv_path, workload, V, T, n_valid, n_params, command):
         "V": V,
         "kernels": kernels,
     }
-    path = os.path.join(ROOT, "profiles", "traffic_per_unit.json")
     with open(path, "w") as f:
         json.dump(out, f, indent=1)
         f.write("\n")
