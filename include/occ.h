@@ -130,7 +130,8 @@ typedef struct {
  * proxy pi_prox of Eq. 5 / pi_async of Table 1).
  *
  *   logits   [T, ld] row-major, dtype dt (bf16 or f32); only columns [0, V) are read
- *   T, V, ld T >= 0 rows, V >= 1 columns, row stride ld >= V (elements)
+ *   T, V, ld T >= 0 rows, 1 <= V <= 2^31 - 1 columns (ids are int32; a larger
+ *            V is OCC_ERR_UNSUPPORTED), row stride ld >= V (elements)
  *   ids      [T] int32 sampled token ids
  *   logp_out [T] float32 (written); NaN where ids[t] is outside [0, V)
  *   lse_out  [T] float32 or NULL

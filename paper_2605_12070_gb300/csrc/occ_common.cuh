@@ -169,6 +169,57 @@ __device__ __forceinline__ void acc_add_fast(LseAcc& a, const float (&x)[N]) {
     acc_add(a, x);
 }
 
+// ------------------------------------------------------------ row streaming
+
+// How a thread walks the vectors i = t, t + NT, t + 2 NT, ... < n of a row,
+// U loads in flight per round.  The shapes differ only in the last, partial
+// round (fewer than U vectors left for the thread):
+//   kSerialTail  the partial round takes one load at a time (each waits for
+//                the previous vector's use: its latency is paid per vector);
+//   kTailRound   full rounds as above, then one round whose loads all issue
+//                together, loads past the row's end repeating the last vector
+//                (in bounds, from L2) and left unused;
+//   kClampAll    every round is that clamped round.
+// Which one is fastest depends on the kernel and its CTA size (GB300
+// measurements at the launch sites).  Row-local indices are 32-bit: V < 2^31.
+enum class Walk { kSerialTail, kTailRound, kClampAll };
+
+// `load(j)` returns the data of vector j (any copyable type), `use(j, d)`
+// consumes it.
+template <Walk W, int U, int NT, typename Load, typename Use>
+__device__ __forceinline__ void walk_row(int t, int n, Load load, Use use) {
+  using D = decltype(load(0));
+  if constexpr (W == Walk::kClampAll) {
+    for (int i = t; i < n; i += U * NT) {
+      D r[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) r[u] = load(min(i + u * NT, n - 1));
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i + u * NT < n) use(i + u * NT, r[u]);
+    }
+  } else {
+    int i = t;
+    for (; i + (U - 1) * NT < n; i += U * NT) {
+      D r[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) r[u] = load(i + u * NT);
+#pragma unroll
+      for (int u = 0; u < U; ++u) use(i + u * NT, r[u]);
+    }
+    if constexpr (W == Walk::kSerialTail) {
+      for (; i < n; i += NT) use(i, load(i));
+    } else if (U > 1 && i < n) {
+      D r[U > 1 ? U - 1 : 1];
+#pragma unroll
+      for (int u = 0; u < U - 1; ++u) r[u] = load(min(i + u * NT, n - 1));
+#pragma unroll
+      for (int u = 0; u < U - 1; ++u)
+        if (i + u * NT < n) use(i + u * NT, r[u]);
+    }
+  }
+}
+
 // ------------------------------------------------------------ reductions
 
 // Two-float compensated addition (Knuth TwoSum on the high parts).

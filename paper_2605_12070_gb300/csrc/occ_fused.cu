@@ -18,6 +18,11 @@
 
 namespace occ {
 
+// One 16-byte vector of the current row and the old row.
+struct RowPair {
+  uint4 t, o;
+};
+
 // Vector path: 16-byte rows.  U vectors of each row in flight per thread.
 // PEEL: rows that start off a 16-byte boundary take their first `lead`
 // elements (up to the boundary) as scalars; the old-logits and gradient rows
@@ -87,18 +92,16 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
       accv_add<1, DIAG>(acc[0], x1, x1);
       accv_add<1, DIAG>(acc[1], xo1, d1);
     };
-    int64_t i = tid;
-    for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
-      uint4 rt[U], ro[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        rt[u] = ld_hint_v4(zv + i + u * NT, keep);
-        ro[u] = ld_hint_v4(zov + i + u * NT, last);
-      }
-#pragma unroll
-      for (int u = 0; u < U; ++u) consume(i + u * NT, rt[u], ro[u]);
-    }
-    for (; i < nvec; i += NT) consume(i, ld_hint_v4(zv + i, keep), ld_hint_v4(zov + i, last));
+    // Row walk (GB300, bf16): clamped rounds in the 128-thread tier (V = 32000:
+    // 2.03 -> 1.99 ms; 24000: 1.76 -> 1.64 ms) and for peeled rows (V = 50257:
+    // 1.94 -> 1.89 ms); one load at a time in the last round for the 256- and
+    // 512-thread tiers of aligned rows (V = 50000: 1.82 against 1.84 ms;
+    // 151936: 8.28-8.31 ms either way).
+    constexpr Walk kW = (NT == 128 || PEEL) ? Walk::kClampAll : Walk::kSerialTail;
+    walk_row<kW, U, NT>(
+        tid, (int)nvec,
+        [&](int j) { return RowPair{ld_hint_v4(zv + j, keep), ld_hint_v4(zov + j, last)}; },
+        [&](int j, const RowPair& r) { consume(j, r.t, r.o); });
     float xt = 0.f, xp = 0.f;
     if ((int64_t)tid < ntail) {
       xt = Elem<Tin>::load(z + tail0 + tid);
@@ -139,15 +142,10 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
         const int64_t nre = nvec - head;
-        int64_t k = tid;
-        for (; k + (int64_t)(2 * U - 1) * NT < nre; k += (int64_t)2 * U * NT) {
-          uint4 r[2 * U];
-#pragma unroll
-          for (int u = 0; u < 2 * U; ++u) r[u] = ld_hint_v4(zv + (head + (k + u * NT)), last);
-#pragma unroll
-          for (int u = 0; u < 2 * U; ++u) emit(head + (k + u * NT), r[u]);
-        }
-        for (; k < nre; k += NT) emit(head + k, ld_hint_v4(zv + (head + k), last));
+        const uint4* zr = zv + head;
+        walk_row<kW, 2 * U, NT>(
+            tid, (int)nre, [&](int j) { return ld_hint_v4(zr + j, last); },
+            [&](int j, const uint4& r) { emit(head + j, r); });
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
         if ((int64_t)tid < ntail) {

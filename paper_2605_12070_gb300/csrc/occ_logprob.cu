@@ -6,6 +6,7 @@
 // U vectors in flight per thread, and keeps an online (c, s) pair per thread;
 // nothing is staged in shared memory because each element is used once.
 // HBM traffic is the logits row once: V * sizeof(T) bytes per token.
+#include <algorithm>
 #include <cstdlib>
 
 #include "occ_common.cuh"
@@ -41,23 +42,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT)
     LseAcc acc;
     acc_init(acc);
     const uint4* zv = reinterpret_cast<const uint4*>(z);
-    int64_t i = threadIdx.x;
-    for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
-      uint4 r[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u) r[u] = ld_stream_v4(zv + i + u * NT);
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        float x[VEC];
-        Elem<Tin>::unpack(r[u], x);
-        acc_add(acc, x);
-      }
-    }
-    for (; i < nvec; i += NT) {
-      float x[VEC];
-      Elem<Tin>::unpack(ld_stream_v4(zv + i), x);
-      acc_add(acc, x);
-    }
+    // Row walk: full rounds, then one round whose loads issue together (GB300:
+    // 0.652 -> 0.603 ms at V = 32000 bf16 against one load at a time).
+    walk_row<Walk::kTailRound, U, NT>(
+        threadIdx.x, (int)nvec, [&](int j) { return ld_stream_v4(zv + j); },
+        [&](int, const uint4& r) {
+          float x[VEC];
+          Elem<Tin>::unpack(r, x);
+          acc_add(acc, x);
+        });
     if ((int64_t)threadIdx.x < V - lead - tail0) {
       float x[1] = {Elem<Tin>::load(z + tail0 + threadIdx.x)};
       acc_add(acc, x);
@@ -75,6 +68,58 @@ __global__ void __launch_bounds__(NT, 1024 / NT)
       if (lse_out) lse_out[row] = (float)l;
     }
     __syncthreads();
+  }
+}
+
+// One warp per row: the same streaming pass, merged with warp shuffles only,
+// so a row costs no CTA barrier and the lane-0 epilogue stalls one warp, not a
+// whole CTA.  Rows are dealt to warps round-robin over the grid.
+template <typename Tin, int NT, int U, bool PEEL>
+__global__ void __launch_bounds__(NT, 1024 / NT)
+    k1_logprob_warp(const Tin* __restrict__ logits, int64_t T, int64_t V, int64_t ld,
+                    const int32_t* __restrict__ ids, float* __restrict__ logp,
+                    float* __restrict__ lse_out) {
+  constexpr int VEC = Elem<Tin>::kVec;
+  constexpr int NW = NT / 32;
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = (int64_t)blockIdx.x * NW + (threadIdx.x >> 5);
+  const int64_t nwarps = (int64_t)gridDim.x * NW;
+  for (int64_t row = warp0; row < T; row += nwarps) {
+    const Tin* z0 = logits + row * ld;
+    const int64_t lead =
+        PEEL ? min(V, (int64_t)(((16 - ((uintptr_t)z0 & 15)) & 15) / sizeof(Tin))) : 0;
+    const Tin* z = z0 + lead;  // 16-byte aligned
+    const int64_t nvec = (V - lead) / VEC;
+    const int64_t tail0 = nvec * VEC;  // relative to z
+    LseAcc acc;
+    acc_init(acc);
+    const uint4* zv = reinterpret_cast<const uint4*>(z);
+    walk_row<Walk::kTailRound, U, 32>(
+        lane, (int)nvec, [&](int j) { return ld_stream_v4(zv + j); },
+        [&](int, const uint4& r) {
+          float x[VEC];
+          Elem<Tin>::unpack(r, x);
+          acc_add(acc, x);
+        });
+    if ((int64_t)lane < V - lead - tail0) {
+      float x[1] = {Elem<Tin>::load(z + tail0 + lane)};
+      acc_add(acc, x);
+    }
+    if (PEEL && (int64_t)lane < lead) {
+      float x[1] = {Elem<Tin>::load(z0 + lane)};
+      acc_add(acc, x);
+    }
+    const float C = warp_max(acc.c);
+    const float2 S = warp_pair_sum(
+        make_float2((acc.c == -INFINITY) ? 0.f : acc.s * exp2f(acc.c - C), 0.f));
+    if (lane == 0) {
+      const int id = ids[row];
+      const bool ok = id >= 0 && id < V;
+      const float zy = ok ? Elem<Tin>::load(z0 + id) : 0.f;
+      const double l = lse_from(C, S);
+      logp[row] = ok ? (float)((double)zy - l) : __int_as_float(0x7fc00000);
+      if (lse_out) lse_out[row] = (float)l;
+    }
   }
 }
 
@@ -125,12 +170,30 @@ static void launch_k1(const void* logits, int64_t T, int64_t V, int64_t ld, cons
     return e ? atoi(e) : 0;
   }();
   if (vec || V >= 16 * Elem<Tin>::kVec) {
-    // rows up to ~96 KB: 128 threads; longer rows: 256 (measured on GB300 from
-    // V = 32000 to 151936 bf16; 512 threads left 2-50 % on the table).  Rows
-    // that are not 16-byte aligned run peeled (scalar head and tail).
+    // Row-size tiers (measured on GB300, V = 4096 to 151936): rows up to 32 KB
+    // one warp each (V = 8192 bf16: 0.64 against 0.88 ms with 128-thread CTAs:
+    // short rows spend much of a CTA's time in its barriers), then CTAs of 128
+    // threads up to ~96 KB and 256 beyond (512 left 2-50 % on the table).
+    // Rows that are not 16-byte aligned run peeled (scalar head and tail).
+    // OCC_K1_WARP (1 / 0) and OCC_K1_THREADS override.
     const int64_t row_bytes = (V / Elem<Tin>::kVec) * 16;
     const int nt = nt_env ? nt_env : (row_bytes <= 96 * 1024 ? 128 : 256);
     const Tin* z = (const Tin*)logits;
+    static const int warp_env = [] {
+      const char* e = getenv("OCC_K1_WARP");
+      return e ? atoi(e) : -1;
+    }();
+    if (warp_env == 1 || (warp_env < 0 && row_bytes <= 32 * 1024)) {
+      constexpr int NTW = 256;  // 8 warps, 4 CTAs per SM
+      const int64_t want = (T + NTW / 32 - 1) / (NTW / 32);
+      const unsigned gw = (unsigned)std::min<int64_t>(want, (int64_t)sm_count() * (1024 / NTW));
+      note_kernel(vec ? "k1_logprob_warp" : "k1_logprob_warp/peel");
+      if (vec)
+        k1_logprob_warp<Tin, NTW, kK1Unroll, false><<<gw, NTW, 0, s>>>(z, T, V, ld, ids, logp, lse);
+      else
+        k1_logprob_warp<Tin, NTW, kK1Unroll, true><<<gw, NTW, 0, s>>>(z, T, V, ld, ids, logp, lse);
+      return;
+    }
 #define OCC_K1_LAUNCH(NT_, PEEL_) \
   k1_logprob_vec<Tin, NT_, kK1Unroll, PEEL_><<<grid, NT_, 0, s>>>(z, T, V, ld, ids, logp, lse)
     note_kernel(vec ? "k1_logprob_vec" : "k1_logprob_vec/peel");
@@ -161,6 +224,8 @@ extern "C" occ_status occ_token_logprob(const void* logits, occ_dtype dt, int64_
   if (T < 0 || V < 1 || ld < V)
     return fail(OCC_ERR_INVALID_ARG, "need T >= 0, V >= 1, ld >= V (T=%lld V=%lld ld=%lld)",
                 (long long)T, (long long)V, (long long)ld);
+  if (V > 0x7fffffffLL)  // token ids are int32; row-local indices are 32-bit
+    return fail(OCC_ERR_UNSUPPORTED, "V = %lld exceeds 2^31 - 1", (long long)V);
   if (T == 0) return OCC_OK;
   if (!logits || !ids || !logp_out) return fail(OCC_ERR_INVALID_ARG, "null logits/ids/logp_out");
   const size_t es = dtype_size(dt);

@@ -608,27 +608,21 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
     const uint4* zv = reinterpret_cast<const uint4*>(z);
     LseAcc acc;
     acc_init(acc);
-    int64_t i = tid;
-    for (; i + (int64_t)(U - 1) * NT < nvec; i += (int64_t)U * NT) {
-      uint4 r[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + i + u * NT, keep);
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int64_t ii = i + u * NT;
-        if (ii < head) head_sm[ii] = r[u];
-        float x[VEC];
-        Elem<Tin>::unpack(r[u], x);
-        acc_add_fast(acc, x);
-      }
-    }
-    for (; i < nvec; i += NT) {
-      const uint4 r = ld_hint_v4(zv + i, keep);
-      if (i < head) head_sm[i] = r;
-      float x[VEC];
-      Elem<Tin>::unpack(r, x);
-      acc_add_fast(acc, x);
-    }
+    // Row walk (GB300, bf16, against one load at a time in the last round):
+    // clamped rounds in the 128- and 512-thread tiers (V = 151936: 6.31 -> 5.93
+    // ms; 32000: 1.48 -> 1.37 ms; 24000: 1.34 -> 1.18 ms), one load at a time
+    // in the 256-thread tier (V = 50000: 1.30 against 1.33 ms) and for peeled
+    // rows (V = 50257: 1.32 against 1.35 ms).
+    constexpr Walk kW = (PEEL || NT == 256) ? Walk::kSerialTail : Walk::kClampAll;
+    const int nh = (int)head;
+    walk_row<kW, U, NT>(
+        tid, (int)nvec, [&](int j) { return ld_hint_v4(zv + j, keep); },
+        [&](int j, const uint4& r) {
+          if (j < nh) head_sm[j] = r;
+          float x[VEC];
+          Elem<Tin>::unpack(r, x);
+          acc_add_fast(acc, x);
+        });
     float xt = 0.f, xp = 0.f;
     if ((int64_t)tid < ntail) {
       xt = Elem<Tin>::load(z + tail0 + tid);
@@ -684,15 +678,10 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
         };
         // re-read part, oldest first: vectors head+tid, head+tid+NT, ... < nvec
         const int64_t nre = nvec - head;
-        int64_t k = tid;
-        for (; k + (int64_t)(U - 1) * NT < nre; k += (int64_t)U * NT) {
-          uint4 r[U];
-#pragma unroll
-          for (int u = 0; u < U; ++u) r[u] = ld_hint_v4(zv + (head + (k + u * NT)), last);
-#pragma unroll
-          for (int u = 0; u < U; ++u) emit(head + (k + u * NT), r[u]);
-        }
-        for (; k < nre; k += NT) emit(head + k, ld_hint_v4(zv + (head + k), last));
+        const uint4* zr = zv + head;
+        walk_row<kW, U, NT>(
+            tid, (int)nre, [&](int j) { return ld_hint_v4(zr + j, last); },
+            [&](int j, const uint4& r) { emit(head + j, r); });
         // on-chip head
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);

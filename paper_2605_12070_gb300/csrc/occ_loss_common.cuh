@@ -410,6 +410,8 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   if (T < 0 || V < 1 || ld < V)
     return fail(OCC_ERR_INVALID_ARG, "need T >= 0, V >= 1, ld >= V (T=%lld V=%lld ld=%lld)",
                 (long long)T, (long long)V, (long long)ld);
+  if (V > 0x7fffffffLL)  // token ids are int32; row-local indices are 32-bit
+    return fail(OCC_ERR_UNSUPPORTED, "V = %lld exceeds 2^31 - 1", (long long)V);
   if (!(p->rd_lo >= 0.0) || !(p->rd_hi >= p->rd_lo) || !(p->eps_low >= 0.0) ||
       !(p->eps_low <= 1.0) || !(p->eps_high >= 0.0) || !isfinite(p->grad_scale) ||
       (p->rd_weight != 0 && p->rd_weight != 1) || (p->dlogits_f32 != 0 && p->dlogits_f32 != 1) ||

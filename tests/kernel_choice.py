@@ -2,7 +2,7 @@
 (row stride V, base address 16-byte aligned), as occ_last_kernel() names it:
 the vector kernel when rows start on 16-byte boundaries, the peeled vector
 kernel when they do not but a row holds at least 16 vectors, else the
-element-load kernel."""
+element-load kernel; for K1, rows of up to 32 KB run one warp per row."""
 
 
 def expected_kernel(kind, V, elem_size):
@@ -10,6 +10,9 @@ def expected_kernel(kind, V, elem_size):
     names = {"k1": ("k1_logprob_vec", "k1_logprob_scalar"),
              "k2": ("k2_loss_l2", "k2_loss_stream"),
              "fused": ("k2_fused_l2", "k2_fused_stream")}[kind]
+    first = names[0]
+    if kind == "k1" and (V // vec) * 16 <= 32 * 1024:  # K1 rows up to 32 KB: one warp each
+        first = "k1_logprob_warp"
     if (V * elem_size) % 16 == 0:
-        return names[0]
-    return names[0] + "/peel" if V >= 16 * vec else names[1]
+        return first
+    return first + "/peel" if V >= 16 * vec else names[1]

@@ -64,12 +64,13 @@ def test_strided_and_misaligned_rows(dtype):
     g = torch.Generator(device="cuda").manual_seed(7)
     big = (torch.randn((9, 5000), generator=g, device="cuda") * 2).to(dtype)
     ids = torch.randint(0, 4097, (9,), generator=g, device="cuda", dtype=torch.int32)
+    vec_kernel = expected_kernel("k1", 4096, big.element_size())  # the aligned-row kernel
     _check(big[:, :4097], ids)        # ld = 5000 > V: aligned rows
-    assert occ.occ_last_kernel() == "k1_logprob_vec"
+    assert occ.occ_last_kernel() == vec_kernel
     _check(big[:, 1:4098], ids)       # base offset by one element: peeled rows
-    assert occ.occ_last_kernel() == "k1_logprob_vec/peel"
+    assert occ.occ_last_kernel() == vec_kernel + "/peel"
     _check(big.reshape(-1)[: 9 * 4097].view(9, 4097), ids)  # ld = V = 4097: peeled rows
-    assert occ.occ_last_kernel() == "k1_logprob_vec/peel"
+    assert occ.occ_last_kernel() == vec_kernel + "/peel"
     _check(big[:, 1:51], ids % 50)    # too short to peel: element loads
     assert occ.occ_last_kernel() == "k1_logprob_scalar"
 
@@ -83,7 +84,8 @@ def test_misaligned_rows_take_the_peeled_vector_kernel(dtype, V):
     ids = torch.randint(0, V, (17,), generator=g, device="cuda", dtype=torch.int32)
     ids[0], ids[-1] = 0, V - 1             # row 0's scalar prefix, the last row's tail
     _check(z, ids)
-    assert occ.occ_last_kernel() == "k1_logprob_vec/peel"
+    assert occ.occ_last_kernel() == expected_kernel("k1", V, z.element_size())
+    assert occ.occ_last_kernel().endswith("/peel")
 
 
 def test_bad_ids_give_nan_and_empty():

@@ -55,6 +55,10 @@ def test_host_validation_without_gpu(L):
     assert L.occ_last_kernel() == b""
     # bad dtype
     assert L.occ_token_logprob(null, 7, 1, 10, 10, null, null, null, null) == 2
+    # a vocabulary that int32 ids cannot index
+    big = 2 ** 31
+    assert L.occ_token_logprob(null, 1, 1, big, big, null, null, null, null) == 2
+    assert b"exceeds" in L.occ_last_error()
     # inverted band
     p = occ.LossParams(2.0, 1.0, 0.2, 0.28, 1.0, 0, 1, 0)
     rc = L.occ_decoupled_loss_fwd_bwd(null, 1, 1, 8, 8, null, null, null, null, null,
