@@ -2,9 +2,10 @@
 //
 // log pi(y_t) = z[t, y_t] - log sum_v exp(z[t, v]) for each row t: the per-token
 // factors of the ratios in Eq. 1 (used for pi_old, pi_prox of Eq. 5 or
-// pi_async of Table 1).  One CTA streams one row with 16-byte coalesced loads,
-// U vectors in flight per thread, and keeps an online (c, s) pair per thread;
-// nothing is staged in shared memory because each element is used once.
+// pi_async of Table 1).  One CTA (or, for rows of up to 32 KB, one warp)
+// streams one row with 16-byte coalesced loads, U vectors in flight per
+// thread, and keeps an online (c, s) pair per thread; nothing is staged in
+// shared memory because each element is used once.
 // HBM traffic is the logits row once: V * sizeof(T) bytes per token.
 #include <algorithm>
 #include <cstdlib>
