@@ -246,7 +246,8 @@ def test_fused_odd_vocab_past_2_31_logits_sampled():
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 20000, 50000, 65536 + 3])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 8184, 8192, 8200, 16376,
+                               16384, 16392, 20000, 50000, 65536, 65536 + 3, 65544])
 def test_fused_vocab_edges(V, dtype):
     # rows shorter than one vector, one vector exactly, a ragged tail after the
     # vector body, rows in each CTA-size tier (40 / 80 / 100 / 200 KB) and rows

@@ -48,8 +48,8 @@ def test_workloads_reduced(name, T):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 31, 63, 65, 127, 129, 4095, 4097, 20000, 50000,
-                               151936])
+@pytest.mark.parametrize("V", [1, 2, 7, 8, 9, 31, 63, 65, 127, 129, 2040, 2048, 2056, 4095, 4097,
+                               16376, 16384, 16392, 20000, 50000, 151936])
 def test_vocab_edges(V, dtype):
     g = torch.Generator(device="cuda").manual_seed(V)
     T = 5

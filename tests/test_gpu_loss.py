@@ -226,8 +226,13 @@ def _edge_batch(T, V, dtype, seed, mask_p=0.8, ld=None, offset=0):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-@pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 20000, 50000, 65536 + 3])
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 63, 65, 127, 129, 4095, 4097, 8184, 8192, 8200, 16376,
+                               16384, 16392, 20000, 50000, 65536, 65536 + 3, 65544])
 def test_vocab_edges(V, dtype):
+    # besides the ragged and tiny rows: rows of one vector less, exactly and
+    # one vector more than whole rounds of loads (forward and re-read, 128- and
+    # 512-thread tiers), where the last partial round of a row is empty or
+    # holds a single vector
     T = 37
     b, lp_old64 = _edge_batch(T, V, dtype, seed=V)
     lp_th64, lse = logprob_rows(b.z_theta, b.ids, np.arange(T))
