@@ -31,10 +31,22 @@ def global_token_count(n_local, group=None):
     return int(t.item())
 
 
+def _allreduce_bits_or(word, group=None):
+    """Bitwise OR of a 32-bit word over ranks, in place.  NCCL has no bitwise
+    reduction, so each bit becomes a 0/1 indicator, the indicators are
+    MAX-reduced, and the word is rebuilt: bit k is set iff some rank set it."""
+    shifts = torch.arange(32, dtype=torch.int64, device=word.device)
+    bits = (word.to(torch.int64) >> shifts) & 1
+    dist.all_reduce(bits, op=dist.ReduceOp.MAX, group=group)
+    packed = (bits << shifts).sum()
+    word.copy_(torch.where(packed >= 2 ** 31, packed - 2 ** 32, packed).to(torch.int32).view(1))
+
+
 def allreduce_loss_stats(stats, group=None):
-    """In-place sum of loss_sum, loss and the four counters over ranks; err is
-    OR-ed (max).  ``denom`` is left as is: every rank must have used the same
-    global denominator."""
+    """In-place sum of loss_sum, loss and the four counters over ranks; the
+    err bits are OR-ed (a rank's BAD_ID and another's TIMEOUT both survive).
+    ``denom`` is left as is: every rank must have used the same global
+    denominator."""
     if stats.dtype != torch.uint8 or stats.numel() != 64:
         raise ValueError("stats must be the 64-byte occ_loss_stats tensor")
     f64 = stats.view(torch.float64)
@@ -42,5 +54,5 @@ def allreduce_loss_stats(stats, group=None):
     i32 = stats.view(torch.int32)
     dist.all_reduce(f64[_F64_LOSS], group=group)
     dist.all_reduce(i64[_I64_COUNTS], group=group)
-    dist.all_reduce(i32[_I32_ERR], op=dist.ReduceOp.MAX, group=group)
+    _allreduce_bits_or(i32[_I32_ERR], group=group)
     return stats

@@ -25,7 +25,7 @@ LIB_PATH = os.path.join(_HERE, "libocc.so")
 OCC_OK = 0
 OCC_F32, OCC_BF16 = 0, 1
 FLAG_IN_BAND, FLAG_CLIPPED, FLAG_ACTIVE, FLAG_VALID = 1, 2, 4, 8
-DATA_ERR_BAD_ID = 1
+DATA_ERR_BAD_ID, DATA_ERR_TIMEOUT = 1, 2
 
 LOSS_STATS_BYTES = 64     # sizeof(occ_loss_stats)
 EWMA_STATE_BYTES = 40     # sizeof(occ_ewma_state)
