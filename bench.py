@@ -255,6 +255,21 @@ def traffic_bytes(tr, name, T, n_valid, n_params):
 
 # ----------------------------------------------------------------- the oracle arm
 
+_EWMA_SAMPLE = {}
+
+
+def _ewma_sample(n):
+    """Host EWMA buffers of n elements (drawn once per size; theta ~ N(0, 0.02^2),
+    theta_prox = theta + N(0, 1e-4^2), like the device buffers)."""
+    if n not in _EWMA_SAMPLE:
+        import torch
+        g = torch.Generator().manual_seed(0)
+        th = (0.02 * torch.randn(n, generator=g)).numpy()
+        _EWMA_SAMPLE.clear()
+        _EWMA_SAMPLE[n] = (th, th + 1e-4 * torch.randn(n, generator=g).numpy())
+    return _EWMA_SAMPLE[n]
+
+
 def oracle_sample_times(batch, rows, n_params, threads):
     """Times the float64 oracle on `rows` tokens and `n_params` EWMA elements.
     Inputs are copied to the host before the clock starts."""
@@ -274,9 +289,7 @@ def oracle_sample_times(batch, rows, n_params, threads):
     adv = batch.adv.cpu().numpy()[rows]
     m = None if mask is None else mask[rows]
     p = oracle.LossParams(**batch.thresholds())
-    g = torch.Generator().manual_seed(0)
-    th = torch.randn(n_params, generator=g).numpy()
-    tp = th + 1e-4 * torch.randn(n_params, generator=g).numpy()
+    th, tp = _ewma_sample(n_params)
     pos = {int(r): k for k, r in enumerate(rows)}
 
     def one(chunk):
@@ -307,43 +320,51 @@ def oracle_sample_times(batch, rows, n_params, threads):
     return t_rows, t_par
 
 
-# Oracle timing calls: tokens and EWMA elements per call, shared by the
-# cpu_baseline leg and the reference arm (small calls are dominated by the
-# thread pool and by numpy's per-array overhead).
-REF_SAMPLE_ROWS = 512
-REF_SAMPLE_PARAMS = 1 << 26
+# One oracle step: REF_SAMPLE_TOKENS tokens drawn from the batch and the same
+# share of the EWMA parameters (n_params x tokens / T), so that the sample has
+# the full step's mix of loss and EWMA work.  Shared by the cpu_baseline leg
+# and the reference arm (smaller calls time the thread pool and numpy's
+# per-array overhead instead of the oracle).
+REF_SAMPLE_TOKENS = 512
 
 
-def cpu_baseline(batch, n_params_full, seconds):
-    """Times the oracle, as it stands, on growing row chunks of the batch and an
-    EWMA sample until about `seconds` of CPU work, then scales to one step."""
+def sample_params(T, n_params_full, tokens=REF_SAMPLE_TOKENS):
+    """EWMA parameters that go with `tokens` of a T-token step."""
+    return max(1, round(n_params_full * tokens / T))
+
+
+def oracle_steps(batch, n_params_full, rng, steps=None, seconds=None):
+    """Runs oracle sample steps (a fixed number, or until `seconds` of work) and
+    returns (tokens per step, params per step, list of step times in s)."""
     import numpy as np
 
     from oracle.rows import host_cores
     threads = host_cores()
-    rng = np.random.default_rng(0)
-    valid = np.nonzero(batch.mask.cpu().numpy())[0] if batch.mask is not None else np.arange(batch.T)
-    order = rng.permutation(valid)
-    t_rows = t_par = 0.0
-    n_rows = n_par = 0
-    chunk = REF_SAMPLE_ROWS  # the reference arm's per-step sample: both time the same calls
-    while t_rows < 0.7 * seconds and n_rows < order.size:
-        rows = np.sort(order[n_rows:n_rows + chunk])
-        tr, _ = oracle_sample_times(batch, rows, 0, threads)
-        t_rows += tr
-        n_rows += rows.size
-    par_chunk = REF_SAMPLE_PARAMS
-    while t_par < 0.3 * seconds and n_par < (1 << 30):
-        _, tp = oracle_sample_times(batch, np.zeros(0, dtype=np.int64), par_chunk, threads)
-        t_par += tp
-        n_par += par_chunk
-    step_s = batch.T * t_rows / n_rows + n_params_full * t_par / n_par
+    S = min(REF_SAMPLE_TOKENS, batch.T)
+    P = sample_params(batch.T, n_params_full, S)
+    times = []
+    while (steps is not None and len(times) < steps) or \
+            (steps is None and sum(times) < seconds):
+        rows = np.sort(rng.choice(batch.T, size=S, replace=False))
+        tr, tp = oracle_sample_times(batch, rows, P, threads)
+        times.append(tr + tp)
+    return S, P, times, threads
+
+
+def cpu_baseline(batch, n_params_full, seconds):
+    """Times the oracle, as it stands, on sample steps of the workload for
+    about `seconds` of work."""
+    import numpy as np
+    S, P, times, threads = oracle_steps(batch, n_params_full, np.random.default_rng(0),
+                                        seconds=seconds)
+    t = sum(times)
     return {
-        "value": round(batch.T / step_s, 3), "unit": "tokens/s", "cores": threads, "kind": "oracle",
-        "sample": (f"float64 numpy oracle on {n_rows} valid tokens of the T={batch.T}, "
-                   f"V={batch.V} batch ({t_rows:.1f} s) and {n_par} EWMA elements "
-                   f"({t_par:.1f} s), scaled to T tokens + {n_params_full} parameters per step"),
-        "seconds": round(t_rows + t_par, 2),
+        "value": round(S * len(times) / t, 3), "unit": "tokens/s", "cores": threads,
+        "kind": "oracle",
+        "sample": (f"{len(times)} oracle steps of {S} tokens drawn from the T={batch.T}, "
+                   f"V={batch.V} batch (log pi_old, loss, dlogits) and {P} EWMA parameters "
+                   f"(the step's parameters-per-token), {t:.1f} s in all, on {threads} threads"),
+        "seconds": round(t, 2),
     }
 
 
@@ -373,9 +394,19 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    if args.impl == "reference" and rank != 0:
+    if args.impl == "reference":
+        # The oracle arm: rank 0 alone, and nothing of the CUDA library (no
+        # build, no libocc.so); the seeded generator only draws the batch.
+        if rank != 0:
+            return
+        from paper_2605_12070_gb300.workloads import make_loss_batch
+        dev = torch.device(f"cuda:{local}" if torch.cuda.is_available() else "cpu")
+        if dev.type == "cuda":
+            torch.cuda.set_device(dev)
+        batch = make_loss_batch(args.workload, T=args.tokens, seed=0, device=dev)
+        run_reference(args, batch, world)
         return
-    if world > 1 and args.impl == "ours":
+    if world > 1:
         torch.cuda.set_device(local)
         dist.init_process_group("nccl")
     dev = torch.device(f"cuda:{local}")
@@ -390,9 +421,6 @@ def main():
     T, V = batch.T, batch.V
     n_valid = T if batch.mask is None else int(batch.mask.sum().item())
 
-    if args.impl == "reference":
-        run_reference(args, batch, world)
-        return
     if args.ewma_variants:
         del batch
         run_ewma_variants(args, dev)
@@ -756,39 +784,52 @@ def workload_config(args, batch, n_valid, world):
 
 
 def run_reference(args, batch, world):
-    """The oracle as the reference arm: each step times the float64 oracle on a
-    bounded sample of the same workload (host cores)."""
+    """The oracle as the reference arm.  Each step is a real, bounded sample of
+    the workload: the float64 oracle on REF_SAMPLE_TOKENS tokens of the batch
+    and the matching share of the EWMA parameters, on the host cores; the
+    line's ms_per_step is the time those steps took, and value is the tokens
+    they processed per second."""
     import numpy as np
 
-    from oracle.rows import host_cores
-    threads = host_cores()
     rng = np.random.default_rng(1)
-    valid = (np.arange(batch.T) if batch.mask is None
-             else np.nonzero(batch.mask.cpu().numpy())[0])
-    rows_n, params_n = min(REF_SAMPLE_ROWS, valid.size), REF_SAMPLE_PARAMS
-    tot_rows = tot_par = 0.0
-    for k in range(args.warmup + args.steps):
-        rows = np.sort(rng.choice(valid, size=rows_n, replace=False))
-        tr, tp = oracle_sample_times(batch, rows, params_n, threads)
-        if k >= args.warmup:
-            tot_rows += tr
-            tot_par += tp
-    step_s = batch.T * (tot_rows / args.steps) / rows_n + args.ewma_n * (tot_par / args.steps) / params_n
-    value = batch.T / step_s
-    sample = (f"per step: float64 oracle on {rows_n} valid tokens of the T={batch.T}, V={batch.V} "
-              f"batch and {params_n} EWMA elements, scaled to the full step")
+    S, P, _, threads = oracle_steps(batch, args.ewma_n, rng, steps=args.warmup)
+    S, P, times, threads = oracle_steps(batch, args.ewma_n, rng, steps=args.steps)
+    step_s = sum(times) / len(times)
+    value = S / step_s
+    n_valid = batch.T if batch.mask is None else int(batch.mask.sum().item())
+    sample = (f"per step: float64 oracle on {S} tokens drawn from the T={batch.T}, V={batch.V} "
+              f"batch (log pi_old, loss, dlogits) and {P} EWMA parameters (the step's "
+              f"parameters-per-token), {threads} threads")
     line = {
         "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(step_s * 1e3, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": dict(workload_config(args, batch, valid.size, world), loss_path="oracle"),
+        "config": dict(workload_config(args, batch, n_valid, world), loss_path="oracle",
+                       sample_tokens_per_step=S, sample_ewma_params_per_step=P),
+        "full_step_s_extrapolated": round(batch.T / value, 2),
         "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": threads,
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
+        "repo_libs_loaded": repo_libs_loaded(),
     }
     print(json.dumps(line), flush=True)
+
+
+def repo_libs_loaded():
+    """Shared objects of this repository mapped into the process (from
+    /proc/self/maps; empty where that file does not exist)."""
+    found = set()
+    try:
+        with open("/proc/self/maps") as f:
+            for line in f:
+                path = line.split()[-1] if len(line.split()) >= 6 else ""
+                if path.startswith(ROOT) and ".so" in os.path.basename(path):
+                    found.add(os.path.relpath(path, ROOT))
+    except OSError:
+        pass
+    return sorted(found)
 
 
 if __name__ == "__main__":

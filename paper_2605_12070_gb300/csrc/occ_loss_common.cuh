@@ -34,8 +34,8 @@ __device__ __forceinline__ double proxy_logprob(int proxy, double alpha, double 
   if (proxy == OCC_PROXY_LOGLINEAR) return alpha * lmu + (1.0 - alpha) * lth;
   const double d = lth - lmu;
   if (d <= 0.0)  // mu >= pi_theta: alpha mu + (1-alpha) pi = mu (1 + (1-alpha) (e^d - 1))
-    return lmu + (double)log1pf((float)(1.0 - alpha) * expm1f((float)d));
-  return lth + (double)log1pf((float)alpha * expm1f((float)-d));
+    return lmu + log1p((1.0 - alpha) * expm1(d));
+  return lth + log1p(alpha * expm1(-d));
 }
 
 struct K2Args {

@@ -85,3 +85,27 @@ def test_shared_workload_config_keys():
     assert cfg["T"] == 8 and cfg["V"] == 16 and "6 valid" in cfg["workload"]
     assert cfg["parallelism"] == "single GPU"
     assert bench.workload_config(A, B, 6, 4)["parallelism"] == "replicas x4"
+
+
+def test_reference_arm_runs_the_oracle_alone(tmp_path):
+    """The oracle arm: no build and no CUDA library in its process, ms_per_step
+    is the time its sample steps took, and value is the tokens they processed
+    per second (nothing extrapolated)."""
+    import json
+    import subprocess
+    import time
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+           "--workload", "tiny_f32_v4096", "--steps", "3", "--warmup", "1",
+           "--ewma-n", "1000000"]
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    t0 = time.time()
+    out = subprocess.run(cmd, capture_output=True, text=True, timeout=300, env=env, cwd=tmp_path)
+    wall = time.time() - t0
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["repo_libs_loaded"] == []
+    S = line["config"]["sample_tokens_per_step"]
+    assert S == 256 and line["config"]["sample_ewma_params_per_step"] == 1000000
+    assert abs(line["value"] - S / (line["ms_per_step"] / 1e3)) <= 1e-3 * line["value"]
+    assert line["steps"] * line["ms_per_step"] / 1e3 < wall
+    assert line["e2e"]["value"] == line["value"] == line["cpu_baseline"]["value"]

@@ -1,0 +1,227 @@
+"""Full-batch parity on the large-vocabulary agentic batch, every token against
+the float64 oracle.
+
+The batch is the one ``bench.py`` times: T = 65536 tokens packed from 128
+sequences (prompt prefixes and padding masked), V = 151936, bf16 logits, band
+[0.8, 1.25], clip 0.2 / 0.28.  The oracle evaluates R1 on all 2 x 65536 rows
+(log pi_theta, log pi_old and both lse), then R2..R9 on all tokens; both loss
+paths of the bench (the fused launch, and K1 followed by K0/K2) are compared
+on every token: log-probabilities (1e-5), flags (bit-exact outside the 1e-6
+threshold exemption, exempt count reported), the four counters and N, and
+the token-mean loss (1e-4 relative; Eqs. 2-4).  dlogits (R8) are compared in
+chunks on more than 2048 rows drawn from every token class: active, clipped,
+out of band, masked, and rows of every class at the batch edges.
+
+The last test chains the 7.6e9-parameter float32 EWMA update (App. B, with
+the auto-reset of Sec. 5.2) on the device statistics of that loss step and
+checks rho, the reset decision, the state and about 3 M sampled parameters
+against the oracle, whose own reset decision comes from its own counters.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from oracle import FLAG_ACTIVE, FLAG_CLIPPED, FLAG_IN_BAND
+from oracle_runner import fp32, logprob_rows, loss_params, oracle_loss
+from oracle.rows import map_row_chunks, to_f64
+from paper_2605_12070_gb300 import occ
+from paper_2605_12070_gb300.workloads import EWMA_N_7B, make_ewma_buffers, make_loss_batch
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+EXEMPT = 1e-6
+LOGP_TIGHT = 1e-5
+LOSS_RTOL = 1e-4
+DZ_ABS = 3e-3
+EWMA_RTOL = 1e-6
+
+
+@pytest.fixture(scope="module")
+def agentic():
+    b = make_loss_batch("agentic_bf16_v151936", seed=0, device="cuda")
+    rows = np.arange(b.T)
+    lo64, _ = logprob_rows(b.z_old, b.ids, rows, chunk=64)
+    lt64, lse = logprob_rows(b.z_theta, b.ids, rows, chunk=64)
+    yield b, lo64, lt64, lse
+    del b
+    torch.cuda.empty_cache()
+
+
+def _dz_rows(o, gfl, T, rng, per_class=512):
+    """At least 2048 rows covering every token class (flag-flipped rows are
+    left out: their gradient depends on the side of the threshold)."""
+    valid = o["valid"]
+    classes = {
+        "active": (o["flags"] & FLAG_ACTIVE) != 0,
+        "clipped": valid & ((o["flags"] & FLAG_CLIPPED) != 0),
+        "out_of_band": valid & ((o["flags"] & FLAG_IN_BAND) == 0),
+        "masked": ~valid,
+    }
+    agree = gfl == o["flags"]
+    pick = [np.array([0, 1, T - 2, T - 1])]
+    for name, sel in classes.items():
+        idx = np.nonzero(sel & agree)[0]
+        assert idx.size > 0, f"the batch has no {name} token"
+        pick.append(rng.choice(idx, size=min(per_class, idx.size), replace=False))
+        pick.append(idx[:4])
+        pick.append(idx[-4:])
+    pick.append(rng.choice(T, size=256, replace=False))
+    rows = np.unique(np.concatenate(pick))
+    rows = rows[agree[rows]]
+    assert rows.size >= 2048, rows.size
+    return rows, classes
+
+
+def _check_dlogits(b, dz, o, lse, rows):
+    """R8 on the given rows, in chunks, against the bf16 dlogits of the GPU."""
+    ids_h = b.ids.cpu().numpy().astype(np.int64)
+
+    def fn(r):
+        it = torch.as_tensor(r, device="cuda")
+        zr = to_f64(b.z_theta[it])
+        ref = orc.softmax_grad_rows(zr, np.clip(ids_h[r], 0, b.V - 1), lse[r], o["g"][r])
+        got = dz[it].float().cpu().numpy().astype(np.float64)
+        g = np.abs(o["g"][r])[:, None]
+        err = np.abs(got - ref)
+        tol = 2.0 ** -8 * np.abs(ref) + 4e-6 * g + 1e-30
+        dead = o["g"][r] == 0.0
+        return (float(err.max()), bool(np.all(err <= tol)), bool(np.all(got[dead] == 0.0)),
+                int(np.count_nonzero(~dead)))
+
+    res = map_row_chunks(fn, rows, chunk=128)
+    assert max(r[0] for r in res) <= DZ_ABS
+    assert all(r[1] for r in res), "dlogits outside the rounding bound"
+    assert all(r[2] for r in res), "a row without gradient is not exactly zero"
+    assert sum(r[3] for r in res) >= 512, "too few compared rows carry a gradient"
+
+
+def _check_every_token(b, out, o, lt64, lo_ref, lo_gpu, exempt_extra=0.0):
+    """Per-token outputs and statistics of one loss call against the oracle."""
+    st = occ.decode_loss_stats(out["stats"])
+    valid = o["valid"]
+    assert st.err == 0
+    assert st.denom == o["N"] and st.n_valid == o["n_valid"] == int(b.mask.sum().item())
+    glp = out["logp"].cpu().numpy().astype(np.float64)
+    assert np.abs(glp[valid] - lt64[valid]).max() <= LOGP_TIGHT
+    assert np.all(glp[~valid] == 0.0)
+    if lo_gpu is not None:
+        assert np.abs(lo_gpu[valid] - lo_ref[valid]).max() <= LOGP_TIGHT
+    gfl = out["flags"].cpu().numpy()
+    near = np.minimum(o["dist_rd"], o["dist_rs"]) <= EXEMPT + exempt_extra
+    diff = gfl != o["flags"]
+    bad = diff & ~(near & valid)
+    assert not bad.any(), (f"{int(bad.sum())} non-exempt flag mismatches at "
+                           f"{np.nonzero(bad)[0][:5]}")
+    nflip = int(diff.sum())
+    print(f"\n  exempt tokens (within {EXEMPT:g} of a threshold): {int((near & valid).sum())}, "
+          f"flag differences among them: {nflip}")
+    counters = (st.n_rd_out, st.n_clipped, st.n_active)
+    ref_counters = (o["n_rd_out"], o["n_clipped"], o["n_active"])
+    if nflip == 0:
+        assert counters == ref_counters
+    else:
+        assert all(abs(x - y) <= nflip for x, y in zip(counters, ref_counters))
+    slack = 0.0
+    if nflip:
+        flipped = diff & (((gfl ^ o["flags"]) & FLAG_IN_BAND) != 0)
+        w = np.maximum(o["r_d"], 1.0)
+        slack = float(np.sum(np.abs(w * o["r_s"] * b.adv.cpu().numpy())[flipped])) / o["N"]
+    assert abs(st.loss - o["loss"]) <= LOSS_RTOL * abs(o["loss"]) + slack, (st.loss, o["loss"])
+    assert abs(st.loss_sum - o["loss_sum"]) <= LOSS_RTOL * abs(o["loss_sum"]) + slack * o["N"]
+    return st, gfl
+
+
+def test_fused_every_token(agentic):
+    """The bench's default path: one launch reads both rows of each token."""
+    b, lo64, lt64, lse = agentic
+    o = oracle_loss(b, lt64, lo64, loss_params(b))   # log pi_old stays float64 in the kernel
+    out = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                       **b.thresholds())
+    torch.cuda.synchronize()
+    assert occ.occ_last_kernel() == "k2_fused_l2"
+    glo = out["logp_old"].cpu().numpy().astype(np.float64)
+    st, gfl = _check_every_token(b, out, o, lt64, lo64, glo)
+    assert np.all(glo[~o["valid"]] == 0.0)
+    # the workload's structure: masked prompts/padding, clipped and out-of-band tokens
+    assert 0 < st.n_rd_out and 0 < st.n_clipped and st.n_valid < b.T
+    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(11))
+    _check_dlogits(b, out["dlogits"], o, lse, rows)
+
+
+def test_two_call_every_token(agentic):
+    """K1 on the old logits, then K0/K2/finalize on the current logits; log
+    pi_old crosses the interface as float32, so the oracle chain rounds its
+    float64 value at the same point."""
+    b, lo64, lt64, lse = agentic
+    lp_old_gpu, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    out = occ.occ_decoupled_loss_fwd_bwd(b.z_theta, b.ids, lp_old_gpu, b.logp_mu, b.adv, b.mask,
+                                         **b.thresholds())
+    torch.cuda.synchronize()
+    assert occ.occ_last_kernel() == "k2_loss_l2"
+    glo = lp_old_gpu.cpu().numpy().astype(np.float64)
+    # K1 reads every row, masked or not: R1 on all 65536 rows
+    assert np.abs(glo - lo64).max() <= LOGP_TIGHT
+    o = oracle_loss(b, lt64, fp32(lo64), loss_params(b))
+    # K1's float32 result may sit one rounding away from the oracle's
+    k1_delta = float(np.abs(glo - fp32(lo64).astype(np.float64)).max())
+    st, gfl = _check_every_token(b, out, o, lt64, None, None, exempt_extra=k1_delta)
+    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(12))
+    _check_dlogits(b, out["dlogits"], o, lse, rows)
+
+
+def _check_ewma(before, th, after, a, b):
+    ref = a * before + b * th
+    scale = np.abs(a * before) + np.abs(b * th)
+    err = np.abs(after.astype(np.float64) - ref)
+    assert np.all(err <= EWMA_RTOL * scale + 1e-30), f"max rel {np.max(err / (scale + 1e-300)):.3g}"
+
+
+def test_ewma_7p6e9_chained_on_the_loss_statistics(agentic):
+    """One fused loss step, then the proximal update of 7.6e9 float32
+    parameters driven by that step's device statistics (no host round trip of
+    rho), three times: tau = 0.9 (the paper's) with min_streak = 2 extends the
+    streak without a reset, the second low step resets theta_prox to theta
+    exactly, and tau = 0.5 then takes a regular update from w = 1."""
+    b, lo64, lt64, _ = agentic
+    o = oracle_loss(b, lt64, lo64, loss_params(b))
+    out = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                       dlogits=None, **b.thresholds())
+    stats = out["stats"]
+    torch.cuda.synchronize()
+    st = occ.decode_loss_stats(stats)
+    rho_ref = o["n_active"] / o["n_valid"]
+    assert abs(st.rho - rho_ref) <= abs(st.n_active - o["n_active"]) / o["n_valid"]
+
+    n, beta = EWMA_N_7B, 0.99
+    th, tp = make_ewma_buffers(n, seed=0, device="cuda")
+    rng = np.random.default_rng(0)
+    idx = np.unique(np.concatenate([rng.integers(0, n, 1_000_000), np.arange(1_000_000),
+                                    np.arange(n - 1_000_000, n)]))
+    it = torch.as_tensor(idx, device="cuda")
+    state = occ.new_ewma_state("cuda", w0=1.0 / (1.0 - beta))
+    ost = orc.EwmaState(w=1.0 / (1.0 - beta))
+    for step, (tau, min_streak) in enumerate([(0.9, 2), (0.9, 2), (0.5, 2)]):
+        assert (rho_ref < tau) == (st.rho < tau), "rho sits between the two counts' ratios"
+        before = tp[it].cpu().numpy().astype(np.float64)
+        thv = th[it].cpu().numpy()
+        occ.occ_ewma_update(tp, th, beta, state, stats=stats, tau=tau, min_streak=min_streak)
+        torch.cuda.synchronize()
+        a, bb, reset, ost = orc.ewma_coefficients(ost, beta, n_active=o["n_active"],
+                                                  n_valid=o["n_valid"], tau=tau,
+                                                  min_streak=min_streak)
+        dst = occ.decode_ewma_state(state)
+        assert (dst.streak, dst.n_resets, bool(dst.last_reset)) == (ost.streak, ost.n_resets,
+                                                                     reset)
+        assert abs(dst.w - ost.w) <= 1e-15 * ost.w
+        assert abs(dst.coef_a - a) <= 1e-15 and abs(dst.coef_b - bb) <= 1e-15
+        after = tp[it].cpu().numpy()
+        if reset:
+            assert np.array_equal(after, thv)
+        else:
+            _check_ewma(before, thv.astype(np.float64), after, a, bb)
+        assert reset == (step == 1)
+        th.add_(1e-4)   # the next actor parameters
+    # the ragged end of the buffer was covered
+    assert idx[-1] == n - 1
