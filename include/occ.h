@@ -19,6 +19,8 @@
  *     host-buffer helpers occ_host_alloc / occ_host_free exist for that).
  *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
  *     default stream).  A returned OCC_OK means the work was enqueued.
+ *     Kernels launch on the current device, which must hold every device
+ *     pointer of the call and the stream.
  *   - Arguments are validated on the host before anything is launched; an
  *     invalid call returns an error status, launches nothing and records a
  *     message readable with occ_last_error() (per host thread).
@@ -229,8 +231,15 @@ occ_status occ_decoupled_loss_fused(const void* logits, const void* logits_old, 
  * every GPU that loads the library holds until the process exits.
  *   - T may be at most OCC_NOALLOC_MAX_TOKENS; larger batches are rejected
  *     with OCC_ERR_UNSUPPORTED before anything is launched.
+ *   - The size limit is checked right after p != NULL and T >= 0, before
+ *     the other arguments.
+ *   - The library uses the scratch array of the CURRENT device, so that
+ *     device must hold the logits and every other pointer and the stream;
+ *     logits on another device are rejected with OCC_ERR_INVALID_ARG.
  *   - The first call on a device (with that device current) looks up the
  *     array's device address; make that first call before any stream capture.
+ *     If the lookup fails, the call returns OCC_ERR_CUDA and the next call
+ *     on that device tries again.
  *   - All calls share the one array: calls that may overlap on the GPU (other
  *     streams, other host threads) race with each other.  Serialise them.
  *     Every call writes all the scratch it later reads, so nothing left over
@@ -338,6 +347,38 @@ occ_status occ_ewma_state_init(occ_ewma_state* st, double w0, void* stream);
 occ_status occ_host_alloc(size_t bytes, void** out);
 occ_status occ_host_free(void* ptr, size_t bytes);
 
+/*
+ * occ_set_option / occ_get_option -- tuning and test controls.  (The paper
+ * has no counterpart: these are measurement plumbing.)
+ *
+ * Every call picks its kernel and launch shape by itself; an option overrides
+ * that choice, for measurements (sweeps of CTA sizes and shared-memory heads,
+ * the alternative kernels) and for the tests of the bounded device waits.
+ * The library reads no environment variable: an option changes only when a
+ * caller sets it.  Options are process-wide and read when a call is launched;
+ * set them between calls.  A value of -1 restores the automatic choice (for
+ * the OCC_OPT_TEST_* controls: off, and the 2 s default limit).
+ * occ_set_option returns OCC_ERR_INVALID_ARG for an unknown option or a value
+ * outside the listed ones; occ_get_option returns -1 for an unknown option.
+ */
+typedef enum {
+  OCC_OPT_K1_WARP = 0,         /* 1: one warp per occ_token_logprob row; 0: CTAs      */
+  OCC_OPT_K1_THREADS = 1,      /* threads per occ_token_logprob CTA: 128, 256, 512   */
+  OCC_OPT_K2_THREADS = 2,      /* threads per occ_decoupled_loss_fwd_bwd CTA: 128, 256, 512 */
+  OCC_OPT_K2_HEAD_BYTES = 3,   /* its shared-memory head, bytes (0 = re-read all from L2) */
+  OCC_OPT_K2_UNROLL = 4,       /* vectors in flight per thread of its 512-thread kernel: 4, 8 */
+  OCC_OPT_FUSED_VARIANT = 5,   /* occ_decoupled_loss_fused: 0 the two-pass kernel,
+                                  1 the persistent TMA-ring kernel                     */
+  OCC_OPT_FUSED_THREADS = 6,   /* threads per two-pass fused CTA: 128, 256, 512       */
+  OCC_OPT_FUSED_HEAD_BYTES = 7, /* its shared-memory head, bytes                       */
+  OCC_OPT_TEST_LOST_COPY_ROW = 8, /* test only: the ring kernel never issues one copy of
+                                  this row, so a wait for it must run out              */
+  OCC_OPT_TEST_WAIT_NS = 9,    /* test only: limit of each bounded device wait, ns (> 0) */
+  OCC_OPT_COUNT_ = 10
+} occ_option;
+occ_status occ_set_option(occ_option opt, int64_t value);
+int64_t occ_get_option(occ_option opt);
+
 /* Static description of a status code. */
 const char* occ_status_string(occ_status s);
 
@@ -345,9 +386,10 @@ const char* occ_status_string(occ_status s);
 const char* occ_last_error(void);
 
 /* The row kernel that the last call on this host thread launched, as a static
- * string: "k1_logprob_vec", "k1_logprob_vec/peel", "k1_logprob_scalar",
- * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_stream", "k2_loss_tma",
- * "k2_loss_reg", "k2_fused_l2", "k2_fused_l2/peel", "k2_fused_stream",
+ * string: "k1_logprob_warp", "k1_logprob_warp/peel", "k1_logprob_vec",
+ * "k1_logprob_vec/peel", "k1_logprob_scalar",
+ * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_stream", "k2_fused_l2",
+ * "k2_fused_l2/peel", "k2_fused_stream",
  * "k2_fused_ring", "k3_ewma_vec", "k3_ewma_scalar", "k3_ewma_bf16" ("" when
  * the call launched none, e.g. T = 0 or an invalid argument).  "/peel" marks
  * the vector kernel run on rows that start off a 16-byte boundary.  Never

@@ -2,6 +2,9 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "occ_internal.h"
 
 namespace occ {
@@ -28,6 +31,37 @@ occ_status check_launch(const char* what) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return fail(OCC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
   return OCC_OK;
+}
+
+static std::atomic<int64_t> g_options[OCC_OPT_COUNT_] = {};
+static std::once_flag g_options_once;
+
+static void options_init() {
+  std::call_once(g_options_once, [] {
+    for (auto& o : g_options) o.store(-1);
+  });
+}
+
+int64_t option(occ_option opt) {
+  options_init();
+  return (opt >= 0 && opt < OCC_OPT_COUNT_) ? g_options[opt].load(std::memory_order_relaxed) : -1;
+}
+
+static bool option_value_ok(occ_option opt, int64_t v) {
+  if (v == -1) return true;
+  switch (opt) {
+    case OCC_OPT_K1_WARP: return v == 0 || v == 1;
+    case OCC_OPT_FUSED_VARIANT: return v == 0 || v == 1;
+    case OCC_OPT_K1_THREADS:
+    case OCC_OPT_K2_THREADS:
+    case OCC_OPT_FUSED_THREADS: return v == 128 || v == 256 || v == 512;
+    case OCC_OPT_K2_UNROLL: return v == 4 || v == 8;
+    case OCC_OPT_K2_HEAD_BYTES:
+    case OCC_OPT_FUSED_HEAD_BYTES: return v >= 0 && v <= 227 * 1024 && v % 16 == 0;
+    case OCC_OPT_TEST_LOST_COPY_ROW: return v >= 0;
+    case OCC_OPT_TEST_WAIT_NS: return v > 0;
+    default: return false;
+  }
 }
 
 int sm_count() {
@@ -80,5 +114,17 @@ const char* occ_last_error(void) { return occ::g_msg; }
 const char* occ_last_kernel(void) { return occ::g_kernel; }
 
 int occ_version(void) { return OCC_VERSION; }
+
+occ_status occ_set_option(occ_option opt, int64_t value) {
+  occ::clear_error();
+  if (opt < 0 || opt >= OCC_OPT_COUNT_ || !occ::option_value_ok(opt, value))
+    return occ::fail(OCC_ERR_INVALID_ARG, "option %d does not take the value %lld", (int)opt,
+                     (long long)value);
+  occ::options_init();
+  occ::g_options[opt].store(value, std::memory_order_relaxed);
+  return OCC_OK;
+}
+
+int64_t occ_get_option(occ_option opt) { return occ::option(opt); }
 
 }  // extern "C"

@@ -237,16 +237,6 @@ __global__ void __launch_bounds__(NT) k2_fused_stream(const FusedArgs f) {
 constexpr int kFusedThreads = 512;
 constexpr int kFusedUnroll = 4;
 
-// OCC_FUSED_VARIANT=ring selects the persistent TMA-ring kernel for the vector
-// path without diagnostics.
-static bool fused_ring_selected() {
-  static const bool v = [] {
-    const char* e = getenv("OCC_FUSED_VARIANT");
-    return e && strcmp(e, "ring") == 0;
-  }();
-  return v;
-}
-
 // The persistent TMA-ring kernel (occ_fused_ring.cu), instantiated there for
 // (bf16, bf16), (bf16, float) and (float, float).
 template <typename Tin, typename Tout>
@@ -283,34 +273,30 @@ template <typename Tin, typename Tout, bool DIAG>
 static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
   const int64_t T = f.a.T;
   const int64_t step = 0x7fffffffLL;
-  if (vec && !DIAG && f.a.V >= Elem<Tin>::kVec && fused_ring_selected())
+  // OCC_OPT_FUSED_VARIANT = 1 selects the persistent TMA-ring kernel for the
+  // vector path without diagnostics.
+  if (vec && !DIAG && f.a.V >= Elem<Tin>::kVec && option(OCC_OPT_FUSED_VARIANT) == 1)
     return launch_fused_ring<Tin, Tout>(f, s);
   const bool peel = !vec && fused_peel_ok<Tin, Tout>(f);
   if (vec || peel) {
-    static const int nt_env = [] {
-      const char* e = getenv("OCC_FUSED_THREADS");
-      return e ? atoi(e) : 0;
-    }();
-    static const long head_env = [] {
-      const char* e = getenv("OCC_FUSED_HEAD_KB");
-      return e ? atol(e) * 1024 : -1L;
-    }();
+    const int64_t nt_opt = option(OCC_OPT_FUSED_THREADS);
+    const int64_t head_opt = option(OCC_OPT_FUSED_HEAD_BYTES);
     // Row-size tiers (measured on GB300, V = 32000 to 151936 bf16): short rows
     // finish in about one load round per CTA, so small CTAs, more of them per
     // SM and no shared-memory head (L2 holds every row in flight) keep the
     // memory system busy; long rows want 512 threads and the largest head
     // with which two CTAs stay in the 164 KB carveout (79 KB for this kernel;
     // at 80 KB it crossed into the 196 KB carveout: 8.38 ms against 8.31 at
-    // V = 151936).
+    // V = 151936).  OCC_OPT_FUSED_THREADS and OCC_OPT_FUSED_HEAD_BYTES override.
     const size_t row_bytes = (size_t)(f.a.V / Elem<Tin>::kVec) * 16;
     const int nt_auto = row_bytes <= 64 * 1024 ? 128 : row_bytes <= 112 * 1024 ? 256 : kFusedThreads;
-    const int nt = nt_env ? nt_env : nt_auto;
+    const int nt = nt_opt > 0 ? (int)nt_opt : nt_auto;
     FusedKern kern = fused_kernel<Tin, Tout, DIAG, false>(nt);
     if constexpr (sizeof(Tin) == sizeof(Tout))
       if (peel) kern = fused_kernel<Tin, Tout, DIAG, true>(nt);
     const size_t head_auto =
         nt_auto == kFusedThreads ? two_cta_smem_budget((const void*)kern) : 0;
-    const size_t head = std::min(head_env >= 0 ? (size_t)head_env : head_auto, row_bytes);
+    const size_t head = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
     f.a.stage_bytes = (int64_t)head;
     if (head > 0) {
       cudaError_t e =

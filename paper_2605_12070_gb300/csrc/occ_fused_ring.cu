@@ -1,5 +1,5 @@
-// Persistent TMA-ring alternative of the fused loss kernel (selected with
-// OCC_FUSED_VARIANT=ring; the default is k2_fused_l2 in occ_fused.cu).
+// Persistent TMA-ring alternative of the fused loss kernel (selected with the
+// option OCC_OPT_FUSED_VARIANT = 1; the default is k2_fused_l2 in occ_fused.cu).
 #include "occ_fused_common.cuh"
 
 namespace occ {
@@ -142,13 +142,17 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
     long long rq = 0;     // row-queue entries pushed
     long long hcount[kHead] = {};  // head copies issued, per head slot
     bool ok = true;
-    auto ring_copy = [&](const void* src, uint32_t bytes, uint64_t pol) -> bool {
+    // `lost` (test hook): the slot is taken but its copy never issued, so the
+    // consumers' wait for it must run out.
+    auto ring_copy = [&](const void* src, uint32_t bytes, uint64_t pol, bool lost) -> bool {
       const int s = (int)(G % kSlots);
       const uint64_t u = G / kSlots;
       if (u >= 1 && !wait(&sh.abort, &sh.empty[s], (uint32_t)((u - 1) & 1), a.wait_ns)) return false;
-      fence_proxy_async_smem();
-      mbar_arrive_expect_tx(&sh.full[s], bytes);
-      bulk_load(slots + (size_t)s * kChunk, src, bytes, &sh.full[s], pol);
+      if (!lost) {
+        fence_proxy_async_smem();
+        mbar_arrive_expect_tx(&sh.full[s], bytes);
+        bulk_load(slots + (size_t)s * kChunk, src, bytes, &sh.full[s], pol);
+      }
       ++G;
       return true;
     };
@@ -177,13 +181,13 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
           bulk_load(head + off, z + off, b, &sh.head_full[k], last);
           ++hcount[k];
         } else {
-          ok = ring_copy(z + off, b, a.dlogits ? keep : last);
+          ok = ring_copy(z + off, b, a.dlogits ? keep : last, false);
         }
-        if (ok) ok = ring_copy(zo + off, b, last);
+        if (ok) ok = ring_copy(zo + off, b, last, k == 0 && row == a.lost_copy_row);
       }
       if (a.dlogits)
         for (int k = nhead; k < nchunk && ok; ++k)
-          ok = ring_copy(z + (size_t)k * kChunk, chunk_bytes(k), last);
+          ok = ring_copy(z + (size_t)k * kChunk, chunk_bytes(k), last, false);
       if (ok) ++jv;
     }
     // drain: every copy issued must land before the CTA's shared memory goes
@@ -399,8 +403,11 @@ __global__ void __launch_bounds__(Gm::kNT, 1) k2_fused_ring(const FusedArgs f) {
 }
 
 template <typename Tin, typename Tout, typename Gm>
-static occ_status launch_fused_ring_geo(const FusedArgs& f, cudaStream_t s) {
+static occ_status launch_fused_ring_geo(FusedArgs f, cudaStream_t s) {
   auto kern = k2_fused_ring<Tin, Tout, Gm>;
+  // test controls of the bounded waits (off unless a test sets them)
+  if (option(OCC_OPT_TEST_LOST_COPY_ROW) >= 0) f.a.lost_copy_row = option(OCC_OPT_TEST_LOST_COPY_ROW);
+  if (option(OCC_OPT_TEST_WAIT_NS) > 0) f.a.wait_ns = (uint64_t)option(OCC_OPT_TEST_WAIT_NS);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)Gm::kSmem);
   if (e != cudaSuccess)

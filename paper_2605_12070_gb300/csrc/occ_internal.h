@@ -27,6 +27,9 @@ inline bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
 
 inline size_t dtype_size(occ_dtype dt) { return dt == OCC_BF16 ? 2 : 4; }
 
+// Current value of a tuning option (occ_set_option); -1 = automatic.
+int64_t option(occ_option opt);
+
 // Multiprocessor count of the current device (cached per device).
 int sm_count();
 

@@ -166,25 +166,19 @@ template <typename Tin>
 static void launch_k1(const void* logits, int64_t T, int64_t V, int64_t ld, const int32_t* ids,
                       float* logp, float* lse, bool vec, cudaStream_t s) {
   const unsigned grid = (unsigned)(T < 0x7fffffffLL ? T : 0x7fffffffLL);
-  static const int nt_env = [] {
-    const char* e = getenv("OCC_K1_THREADS");
-    return e ? atoi(e) : 0;
-  }();
+  const int64_t nt_opt = option(OCC_OPT_K1_THREADS);
   if (vec || V >= 16 * Elem<Tin>::kVec) {
     // Row-size tiers (measured on GB300, V = 4096 to 151936): rows up to 32 KB
     // one warp each (V = 8192 bf16: 0.64 against 0.88 ms with 128-thread CTAs:
     // short rows spend much of a CTA's time in its barriers), then CTAs of 128
     // threads up to ~96 KB and 256 beyond (512 left 2-50 % on the table).
     // Rows that are not 16-byte aligned run peeled (scalar head and tail).
-    // OCC_K1_WARP (1 / 0) and OCC_K1_THREADS override.
+    // The options OCC_OPT_K1_WARP (1 / 0) and OCC_OPT_K1_THREADS override.
     const int64_t row_bytes = (V / Elem<Tin>::kVec) * 16;
-    const int nt = nt_env ? nt_env : (row_bytes <= 96 * 1024 ? 128 : 256);
+    const int nt = nt_opt > 0 ? (int)nt_opt : (row_bytes <= 96 * 1024 ? 128 : 256);
     const Tin* z = (const Tin*)logits;
-    static const int warp_env = [] {
-      const char* e = getenv("OCC_K1_WARP");
-      return e ? atoi(e) : -1;
-    }();
-    if (warp_env == 1 || (warp_env < 0 && row_bytes <= 32 * 1024)) {
+    const int64_t warp_opt = option(OCC_OPT_K1_WARP);
+    if (warp_opt == 1 || (warp_opt < 0 && row_bytes <= 32 * 1024)) {
       constexpr int NTW = 256;  // 8 warps, 4 CTAs per SM
       const int64_t want = (T + NTW / 32 - 1) / (NTW / 32);
       const unsigned gw = (unsigned)std::min<int64_t>(want, (int64_t)sm_count() * (1024 / NTW));

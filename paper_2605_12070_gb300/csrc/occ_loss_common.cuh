@@ -41,11 +41,11 @@ __device__ __forceinline__ double proxy_logprob(int proxy, double alpha, double 
 struct K2Args {
   const void* logits;
   int64_t T, V, ld, S, row0;
-  int64_t stage_bytes;  // shared-memory bytes of one pipeline stage (TMA kernel)
+  int64_t stage_bytes;  // bytes of the shared-memory head of the row (two-pass kernels)
   int* ws_err;          // device-detected error bits, OR-ed into stats.err
-  unsigned long long* ws_rows;  // token counter of the persistent kernels (zeroed by K0)
-  uint64_t wait_ns;     // limit of each wait for an asynchronous copy (cluster kernels)
-  int64_t lost_copy_row;  // test hook (-1 = off): the copy of this row is never issued
+  unsigned long long* ws_rows;  // token counter of the persistent ring kernel (zeroed by K0)
+  uint64_t wait_ns;     // limit of each wait for an asynchronous copy (ring kernel)
+  int64_t lost_copy_row;  // test hook (-1 = off): one copy of this row is never issued
   const int32_t* ids;
   const float* lp_old;
   const float* lp_mu;

@@ -10,6 +10,7 @@ There is no CPU fallback: if the library is missing or a tensor is not on a
 CUDA device, the call raises.
 """
 
+import contextlib
 import ctypes
 import math
 import os
@@ -37,7 +38,12 @@ EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_
            "occ_decoupled_loss_fused", "occ_decoupled_loss_fwd_bwd_noalloc", "occ_ewma_update",
            "occ_ewma_update_bf16", "occ_ewma_update_host", "occ_ewma_state_init",
            "occ_host_alloc", "occ_host_free", "occ_status_string", "occ_last_error",
-           "occ_last_kernel", "occ_version")
+           "occ_last_kernel", "occ_version", "occ_set_option", "occ_get_option")
+
+# occ_option codes (include/occ.h)
+OPTIONS = {"k1_warp": 0, "k1_threads": 1, "k2_threads": 2, "k2_head_bytes": 3, "k2_unroll": 4,
+           "fused_variant": 5, "fused_threads": 6, "fused_head_bytes": 7,
+           "test_lost_copy_row": 8, "test_wait_ns": 9}
 
 
 class OccError(RuntimeError):
@@ -116,8 +122,34 @@ def lib():
     L.occ_last_kernel.restype = ctypes.c_char_p
     L.occ_version.argtypes = []
     L.occ_version.restype = ctypes.c_int
+    L.occ_set_option.argtypes = [i32, i64]
+    L.occ_set_option.restype = i32
+    L.occ_get_option.argtypes = [i32]
+    L.occ_get_option.restype = i64
     _lib = L
     return L
+
+
+def set_option(name, value):
+    """Sets a process-wide tuning or test option (-1 = automatic / off)."""
+    _check(lib().occ_set_option(OPTIONS[name], int(value)), f"occ_set_option({name})")
+
+
+def get_option(name):
+    return int(lib().occ_get_option(OPTIONS[name]))
+
+
+@contextlib.contextmanager
+def options(**kw):
+    """Sets options for the duration of a block, then restores them."""
+    old = {k: get_option(k) for k in kw}
+    try:
+        for k, v in kw.items():
+            set_option(k, v)
+        yield
+    finally:
+        for k, v in old.items():
+            set_option(k, v)
 
 
 def occ_last_kernel():
@@ -139,6 +171,12 @@ def _ptr(t):
 def _stream(stream, device):
     s = stream if stream is not None else torch.cuda.current_stream(device)
     return ctypes.c_void_p(s.cuda_stream)
+
+
+def _on(device):
+    """Makes `device` current for the call: the library launches on the
+    current device, which must hold every pointer and the stream."""
+    return torch.cuda.device(device)
 
 
 def _cuda(*ts):
@@ -169,8 +207,9 @@ def occ_token_logprob(logits, ids, logp_out=None, lse_out=None, want_lse=False, 
         logp_out = torch.empty(T, dtype=torch.float32, device=logits.device)
     if lse_out is None and want_lse:
         lse_out = torch.empty(T, dtype=torch.float32, device=logits.device)
-    rc = lib().occ_token_logprob(_ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids),
-                                 _ptr(logp_out), _ptr(lse_out), _stream(stream, logits.device))
+    with _on(logits.device):
+        rc = lib().occ_token_logprob(_ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids),
+                                     _ptr(logp_out), _ptr(lse_out), _stream(stream, logits.device))
     _check(rc, "occ_token_logprob")
     return logp_out, lse_out
 
@@ -248,11 +287,12 @@ def occ_decoupled_loss_fwd_bwd(logits, ids, logp_old, logp_mu, adv, loss_mask=No
         workspace = new_workspace(T, V, dev)
     p = _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32,
                 proxy, alpha)
-    rc = lib().occ_decoupled_loss_fwd_bwd(
-        _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
-        _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
-        _ptr(dlogits), ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(),
-        _stream(stream, dev))
+    with _on(dev):
+        rc = lib().occ_decoupled_loss_fwd_bwd(
+            _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
+            _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
+            _ptr(dlogits), ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(),
+            _stream(stream, dev))
     _check(rc, "occ_decoupled_loss_fwd_bwd")
     return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "flags": flags_out}
 
@@ -299,11 +339,12 @@ def occ_decoupled_loss_fused(logits, logits_old, ids, logp_mu, adv, loss_mask=No
     if workspace is None:
         workspace = new_workspace(T, V, dev)
     p = _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32)
-    rc = lib().occ_decoupled_loss_fused(
-        _ptr(logits), _ptr(logits_old), _dtype_code(logits), T, V, ld, ld_old, _ptr(ids),
-        _ptr(logp_mu), _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out),
-        _ptr(logp_old_out), _ptr(flags_out), _ptr(entropy_out), _ptr(kl_out), _ptr(dlogits),
-        ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(), _stream(stream, dev))
+    with _on(dev):
+        rc = lib().occ_decoupled_loss_fused(
+            _ptr(logits), _ptr(logits_old), _dtype_code(logits), T, V, ld, ld_old, _ptr(ids),
+            _ptr(logp_mu), _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out),
+            _ptr(logp_old_out), _ptr(flags_out), _ptr(entropy_out), _ptr(kl_out), _ptr(dlogits),
+            ld_grad, _ptr(stats), _ptr(workspace), workspace.numel(), _stream(stream, dev))
     _check(rc, "occ_decoupled_loss_fused")
     return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "logp_old": logp_old_out,
             "flags": flags_out, "entropy": entropy_out, "kl": kl_out}
@@ -327,10 +368,11 @@ def occ_decoupled_loss_fwd_bwd_noalloc(logits, ids, logp_old, logp_mu, adv, loss
     T, V, ld = _rows(logits)
     ld_grad = dlogits.stride(0) if dlogits is not None else 0
     p = _params(rd_lo, rd_hi, eps_low, eps_high, grad_scale, denom, rd_weight, dlogits_f32)
-    rc = lib().occ_decoupled_loss_fwd_bwd_noalloc(
-        _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
-        _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
-        _ptr(dlogits), ld_grad, _ptr(stats), _stream(stream, logits.device))
+    with _on(logits.device):
+        rc = lib().occ_decoupled_loss_fwd_bwd_noalloc(
+            _ptr(logits), _dtype_code(logits), T, V, ld, _ptr(ids), _ptr(logp_old), _ptr(logp_mu),
+            _ptr(adv), _ptr(loss_mask), ctypes.byref(p), _ptr(logp_out), _ptr(flags_out),
+            _ptr(dlogits), ld_grad, _ptr(stats), _stream(stream, logits.device))
     _check(rc, "occ_decoupled_loss_fwd_bwd_noalloc")
     return {"stats": stats, "dlogits": dlogits, "logp": logp_out, "flags": flags_out}
 
@@ -343,8 +385,9 @@ def new_ewma_state(device, w0=0.0, stream=None):
 
 def occ_ewma_state_init(state, w0, stream=None):
     _cuda(state)
-    _check(lib().occ_ewma_state_init(_ptr(state), float(w0), _stream(stream, state.device)),
-           "occ_ewma_state_init")
+    with _on(state.device):
+        rc = lib().occ_ewma_state_init(_ptr(state), float(w0), _stream(stream, state.device))
+    _check(rc, "occ_ewma_state_init")
 
 
 @dataclass
@@ -373,9 +416,10 @@ def occ_ewma_update(theta_prox, theta, beta, state, stats=None, tau=0.9, min_str
     n = theta_prox.numel()
     if theta.numel() != n:
         raise OccError("theta_prox and theta differ in size")
-    rc = lib().occ_ewma_update(_ptr(theta_prox), _ptr(theta), n, float(beta), _ptr(state),
-                               _ptr(stats), float(tau), int(min_streak), int(bool(force_reset)),
-                               _stream(stream, theta_prox.device))
+    with _on(theta_prox.device):
+        rc = lib().occ_ewma_update(_ptr(theta_prox), _ptr(theta), n, float(beta), _ptr(state),
+                                   _ptr(stats), float(tau), int(min_streak), int(bool(force_reset)),
+                                   _stream(stream, theta_prox.device))
     _check(rc, "occ_ewma_update")
     return theta_prox
 
@@ -396,10 +440,11 @@ def occ_ewma_update_bf16(theta_prox, theta, beta, state, stats=None, tau=0.9, mi
     if theta_prox.dtype != torch.bfloat16 or not theta_prox.is_contiguous() or \
             not theta.is_contiguous() or theta.numel() != theta_prox.numel():
         raise OccError("theta_prox must be contiguous bf16 and match theta")
-    rc = lib().occ_ewma_update_bf16(_ptr(theta_prox), _ptr(theta), _float_code(theta),
-                                    theta_prox.numel(), float(beta), _ptr(state), _ptr(stats),
-                                    float(tau), int(min_streak), int(bool(force_reset)),
-                                    int(sr_seed), _stream(stream, theta_prox.device))
+    with _on(theta_prox.device):
+        rc = lib().occ_ewma_update_bf16(_ptr(theta_prox), _ptr(theta), _float_code(theta),
+                                        theta_prox.numel(), float(beta), _ptr(state), _ptr(stats),
+                                        float(tau), int(min_streak), int(bool(force_reset)),
+                                        int(sr_seed), _stream(stream, theta_prox.device))
     _check(rc, "occ_ewma_update_bf16")
     return theta_prox
 
@@ -414,11 +459,12 @@ def occ_ewma_update_host(theta_prox_host, theta, beta, state, staging, stats=Non
     dev = theta.device
     s0 = stream0 if stream0 is not None else torch.cuda.current_stream(dev)
     s1 = stream1 if stream1 is not None else s0
-    rc = lib().occ_ewma_update_host(
-        _ptr(theta_prox_host), _float_code(theta_prox_host), _ptr(theta), _float_code(theta),
-        theta.numel(), float(beta), _ptr(state), _ptr(stats), float(tau), int(min_streak),
-        int(bool(force_reset)), int(sr_seed), _ptr(staging), staging.numel(),
-        ctypes.c_void_p(s0.cuda_stream), ctypes.c_void_p(s1.cuda_stream))
+    with _on(dev):
+        rc = lib().occ_ewma_update_host(
+            _ptr(theta_prox_host), _float_code(theta_prox_host), _ptr(theta), _float_code(theta),
+            theta.numel(), float(beta), _ptr(state), _ptr(stats), float(tau), int(min_streak),
+            int(bool(force_reset)), int(sr_seed), _ptr(staging), staging.numel(),
+            ctypes.c_void_p(s0.cuda_stream), ctypes.c_void_p(s1.cuda_stream))
     _check(rc, "occ_ewma_update_host")
     return theta_prox_host
 

@@ -49,9 +49,10 @@ def agentic():
     torch.cuda.empty_cache()
 
 
-def _dz_rows(o, gfl, T, rng, per_class=512):
-    """At least 2048 rows covering every token class (flag-flipped rows are
-    left out: their gradient depends on the side of the threshold)."""
+def _dz_rows(o, gfl, T, rng, require, per_class=800):
+    """At least 2048 rows covering every token class present (flag-flipped
+    rows are left out: their gradient depends on the side of the threshold);
+    the classes in `require` must be present."""
     valid = o["valid"]
     classes = {
         "active": (o["flags"] & FLAG_ACTIVE) != 0,
@@ -63,7 +64,9 @@ def _dz_rows(o, gfl, T, rng, per_class=512):
     pick = [np.array([0, 1, T - 2, T - 1])]
     for name, sel in classes.items():
         idx = np.nonzero(sel & agree)[0]
-        assert idx.size > 0, f"the batch has no {name} token"
+        assert idx.size > 0 or name not in require, f"the batch has no {name} token"
+        if idx.size == 0:
+            continue
         pick.append(rng.choice(idx, size=min(per_class, idx.size), replace=False))
         pick.append(idx[:4])
         pick.append(idx[-4:])
@@ -144,9 +147,11 @@ def test_fused_every_token(agentic):
     glo = out["logp_old"].cpu().numpy().astype(np.float64)
     st, gfl = _check_every_token(b, out, o, lt64, lo64, glo)
     assert np.all(glo[~o["valid"]] == 0.0)
-    # the workload's structure: masked prompts/padding, clipped and out-of-band tokens
-    assert 0 < st.n_rd_out and 0 < st.n_clipped and st.n_valid < b.T
-    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(11))
+    # the workload's structure: masked prompts and padding, clipped tokens, and no
+    # token outside the band (the rollout noise, sigma = 0.02 in log space, sits
+    # 11 sigma inside log 1.25); the heavy-tailed batch below covers that class
+    assert 0 < st.n_clipped and st.n_valid < b.T and st.n_rd_out == o["n_rd_out"] == 0
+    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(11), ("active", "clipped", "masked"))
     _check_dlogits(b, out["dlogits"], o, lse, rows)
 
 
@@ -167,7 +172,29 @@ def test_two_call_every_token(agentic):
     # K1's float32 result may sit one rounding away from the oracle's
     k1_delta = float(np.abs(glo - fp32(lo64).astype(np.float64)).max())
     st, gfl = _check_every_token(b, out, o, lt64, None, None, exempt_extra=k1_delta)
-    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(12))
+    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(12), ("active", "clipped", "masked"))
+    _check_dlogits(b, out["dlogits"], o, lse, rows)
+
+
+def test_heavytail_every_token_and_every_class():
+    """The heavy-tailed batch (T = 16384, V = 151936, Student-t rollout noise):
+    1-5 % of the tokens fall outside the band, so dlogits are compared on rows
+    of every class, out-of-band ones included, through the fused launch."""
+    b = make_loss_batch("heavytail_bf16_v151936", seed=0, device="cuda")
+    rows = np.arange(b.T)
+    lo64, _ = logprob_rows(b.z_old, b.ids, rows, chunk=64)
+    lt64, lse = logprob_rows(b.z_theta, b.ids, rows, chunk=64)
+    b.mask = torch.ones(b.T, dtype=torch.uint8, device="cuda")
+    b.mask[::7] = 0   # some masked rows, so that every class is present
+    o = oracle_loss(b, lt64, lo64, loss_params(b))
+    out = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                       **b.thresholds())
+    torch.cuda.synchronize()
+    glo = out["logp_old"].cpu().numpy().astype(np.float64)
+    st, gfl = _check_every_token(b, out, o, lt64, lo64, glo)
+    assert 0.01 <= st.n_rd_out / st.n_valid <= 0.05
+    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(13),
+                       ("active", "clipped", "out_of_band", "masked"))
     _check_dlogits(b, out["dlogits"], o, lse, rows)
 
 

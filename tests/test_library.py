@@ -71,6 +71,19 @@ def test_host_validation_without_gpu(L):
                                       ctypes.byref(p), null, null, null, 0,
                                       ctypes.cast(stats, ctypes.c_void_p), null, 0, null)
     assert rc == 5
+    # allocation-free loss: a null params pointer and a negative T are argument
+    # errors before the size limit is looked at; only then is a T beyond the
+    # scratch array unsupported (all before any CUDA call)
+    nf = L.occ_decoupled_loss_fwd_bwd_noalloc
+    big_T = occ.NOALLOC_MAX_TOKENS + 1
+    assert nf(null, 1, big_T, 8, 8, null, null, null, null, null, None, null, null, null, 0,
+              null, null) == 1
+    assert b"params" in L.occ_last_error()
+    assert nf(null, 1, -1, 8, 8, null, null, null, null, null, ctypes.byref(p), null, null, null,
+              0, null, null) == 1
+    assert nf(null, 1, big_T, 8, 8, null, null, null, null, null, ctypes.byref(p), null, null,
+              null, 0, null, null) == 2
+    assert b"at most" in L.occ_last_error()
     # EWMA: beta out of range, min_streak < 1
     st = ctypes.create_string_buffer(48)
     stp = ctypes.cast(st, ctypes.c_void_p)
@@ -174,3 +187,20 @@ def test_concurrent_builds_take_turns():
     L2 = ctypes.CDLL(build.LIB)
     for name in occ.EXPORTS:
         assert hasattr(L2, name), name
+
+
+def test_options_are_explicit_and_checked(L):
+    # the library reads no environment variable: an option changes only through
+    # occ_set_option, rejects values it does not know, and -1 restores the default
+    import os
+    assert "getenv" not in open(os.path.join(os.path.dirname(occ.LIB_PATH), "csrc",
+                                             "occ_loss.cu")).read()
+    for name, code in occ.OPTIONS.items():
+        assert L.occ_get_option(code) == -1, name
+    assert L.occ_set_option(2, 256) == 0 and L.occ_get_option(2) == 256
+    assert L.occ_set_option(2, 300) == 1 and L.occ_get_option(2) == 256
+    assert L.occ_set_option(2, -1) == 0 and L.occ_get_option(2) == -1
+    assert L.occ_set_option(99, 1) == 1 and L.occ_get_option(99) == -1
+    with occ.options(fused_variant=1, test_wait_ns=1000):
+        assert occ.get_option("fused_variant") == 1 and occ.get_option("test_wait_ns") == 1000
+    assert occ.get_option("fused_variant") == -1 and occ.get_option("test_wait_ns") == -1
