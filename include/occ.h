@@ -63,7 +63,6 @@ typedef enum { OCC_F32 = 0, OCC_BF16 = 1 } occ_dtype;
 
 /* Bits of occ_loss_stats.err (device-detected data problems). */
 #define OCC_DATA_ERR_BAD_ID 1 /* some token id was outside [0, V); those tokens were dropped */
-#define OCC_DATA_ERR_TIMEOUT 2 /* a bounded wait for an asynchronous copy gave up; outputs invalid */
 
 /* Bits of the per-token flags written by occ_decoupled_loss_fwd_bwd. */
 #define OCC_FLAG_IN_BAND 1 /* r_d inside [rd_lo, rd_hi]                        (Eq. 4) */
@@ -353,11 +352,10 @@ occ_status occ_host_free(void* ptr, size_t bytes);
  *
  * Every call picks its kernel and launch shape by itself; an option overrides
  * that choice, for measurements (sweeps of CTA sizes and shared-memory heads,
- * the alternative kernels) and for the tests of the bounded device waits.
+ * measurements of the launch shapes.
  * The library reads no environment variable: an option changes only when a
  * caller sets it.  Options are process-wide and read when a call is launched;
- * set them between calls.  A value of -1 restores the automatic choice (for
- * the OCC_OPT_TEST_* controls: off, and the 2 s default limit).
+ * set them between calls.  A value of -1 restores the automatic choice.
  * occ_set_option returns OCC_ERR_INVALID_ARG for an unknown option or a value
  * outside the listed ones; occ_get_option returns -1 for an unknown option.
  */
@@ -367,14 +365,9 @@ typedef enum {
   OCC_OPT_K2_THREADS = 2,      /* threads per occ_decoupled_loss_fwd_bwd CTA: 128, 256, 512 */
   OCC_OPT_K2_HEAD_BYTES = 3,   /* its shared-memory head, bytes (0 = re-read all from L2) */
   OCC_OPT_K2_UNROLL = 4,       /* vectors in flight per thread of its 512-thread kernel: 4, 8 */
-  OCC_OPT_FUSED_VARIANT = 5,   /* occ_decoupled_loss_fused: 0 the two-pass kernel,
-                                  1 the persistent TMA-ring kernel                     */
-  OCC_OPT_FUSED_THREADS = 6,   /* threads per two-pass fused CTA: 128, 256, 512       */
-  OCC_OPT_FUSED_HEAD_BYTES = 7, /* its shared-memory head, bytes                       */
-  OCC_OPT_TEST_LOST_COPY_ROW = 8, /* test only: the ring kernel never issues one copy of
-                                  this row, so a wait for it must run out              */
-  OCC_OPT_TEST_WAIT_NS = 9,    /* test only: limit of each bounded device wait, ns (> 0) */
-  OCC_OPT_COUNT_ = 10
+  OCC_OPT_FUSED_THREADS = 5,   /* threads per occ_decoupled_loss_fused CTA: 128, 256, 512 */
+  OCC_OPT_FUSED_HEAD_BYTES = 6, /* its shared-memory head, bytes                       */
+  OCC_OPT_COUNT_ = 7
 } occ_option;
 occ_status occ_set_option(occ_option opt, int64_t value);
 int64_t occ_get_option(occ_option opt);

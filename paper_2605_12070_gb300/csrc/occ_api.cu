@@ -51,15 +51,12 @@ static bool option_value_ok(occ_option opt, int64_t v) {
   if (v == -1) return true;
   switch (opt) {
     case OCC_OPT_K1_WARP: return v == 0 || v == 1;
-    case OCC_OPT_FUSED_VARIANT: return v == 0 || v == 1;
     case OCC_OPT_K1_THREADS:
     case OCC_OPT_K2_THREADS:
     case OCC_OPT_FUSED_THREADS: return v == 128 || v == 256 || v == 512;
     case OCC_OPT_K2_UNROLL: return v == 4 || v == 8;
     case OCC_OPT_K2_HEAD_BYTES:
     case OCC_OPT_FUSED_HEAD_BYTES: return v >= 0 && v <= 227 * 1024 && v % 16 == 0;
-    case OCC_OPT_TEST_LOST_COPY_ROW: return v >= 0;
-    case OCC_OPT_TEST_WAIT_NS: return v > 0;
     default: return false;
   }
 }

@@ -237,11 +237,6 @@ __global__ void __launch_bounds__(NT) k2_fused_stream(const FusedArgs f) {
 constexpr int kFusedThreads = 512;
 constexpr int kFusedUnroll = 4;
 
-// The persistent TMA-ring kernel (occ_fused_ring.cu), instantiated there for
-// (bf16, bf16), (bf16, float) and (float, float).
-template <typename Tin, typename Tout>
-occ_status launch_fused_ring(const FusedArgs& f, cudaStream_t s);
-
 using FusedKern = void (*)(const FusedArgs);
 
 template <typename Tin, typename Tout, bool DIAG, bool PEEL>
@@ -273,10 +268,6 @@ template <typename Tin, typename Tout, bool DIAG>
 static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
   const int64_t T = f.a.T;
   const int64_t step = 0x7fffffffLL;
-  // OCC_OPT_FUSED_VARIANT = 1 selects the persistent TMA-ring kernel for the
-  // vector path without diagnostics.
-  if (vec && !DIAG && f.a.V >= Elem<Tin>::kVec && option(OCC_OPT_FUSED_VARIANT) == 1)
-    return launch_fused_ring<Tin, Tout>(f, s);
   const bool peel = !vec && fused_peel_ok<Tin, Tout>(f);
   if (vec || peel) {
     const int64_t nt_opt = option(OCC_OPT_FUSED_THREADS);

@@ -1,4 +1,4 @@
-// Shared by the fused loss kernels (occ_fused.cu, occ_fused_ring.cu): their
+// Shared by the fused loss kernels (occ_fused.cu): their
 // arguments and the per-token epilogue that turns the two merged rows into
 // log pi_old, log pi_theta, the Eq. 2-4 decisions and the backward scale.
 #pragma once

@@ -43,9 +43,6 @@ struct K2Args {
   int64_t T, V, ld, S, row0;
   int64_t stage_bytes;  // bytes of the shared-memory head of the row (two-pass kernels)
   int* ws_err;          // device-detected error bits, OR-ed into stats.err
-  unsigned long long* ws_rows;  // token counter of the persistent ring kernel (zeroed by K0)
-  uint64_t wait_ns;     // limit of each wait for an asynchronous copy (ring kernel)
-  int64_t lost_copy_row;  // test hook (-1 = off): one copy of this row is never issued
   const int32_t* ids;
   const float* lp_old;
   const float* lp_mu;
@@ -184,13 +181,9 @@ template <int NT>
 __global__ void __launch_bounds__(NT) k0_count_valid(const uint8_t* __restrict__ mask,
                                                      const int32_t* __restrict__ ids, int64_t T,
                                                      int64_t V, long long* __restrict__ ws_N,
-                                                     int* __restrict__ ws_err,
-                                                     unsigned long long* __restrict__ ws_rows) {
+                                                     int* __restrict__ ws_err) {
   __shared__ long long part[NT / 32];
-  if (threadIdx.x == 0) {
-    *ws_err = 0;
-    *ws_rows = 0;
-  }
+  if (threadIdx.x == 0) *ws_err = 0;
   long long c = 0;
   for (int64_t t0 = threadIdx.x; t0 < T; t0 += 8 * (int64_t)NT) {
     int idv[8];
@@ -287,14 +280,13 @@ __global__ void __launch_bounds__(NT) k2_finalize(int64_t T, const float* __rest
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct WsLayout {
-  size_t off_N, off_err, off_rows, off_loss, off_flags, total;
+  size_t off_N, off_err, off_loss, off_flags, total;
 };
 inline WsLayout ws_layout(int64_t T) {
   const size_t t = T > 0 ? (size_t)T : 0;
   WsLayout w;
   w.off_N = 0;
   w.off_err = 8;
-  w.off_rows = 16;
   w.off_loss = 256;
   w.off_flags = w.off_loss + align_up(4 * t, 256);
   w.total = w.off_flags + align_up(t, 256);
@@ -457,8 +449,6 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   a.S = V;
   a.row0 = 0;
   a.stage_bytes = 0;
-  a.wait_ns = 2000000000ull;
-  a.lost_copy_row = -1;
   a.ids = ids;
   a.lp_old = nullptr;
   a.lp_mu = logp_mu;
@@ -466,7 +456,6 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   a.mask = loss_mask;
   a.ws_N = (const long long*)(ws + wl.off_N);
   a.ws_err = (int*)(ws + wl.off_err);
-  a.ws_rows = (unsigned long long*)(ws + wl.off_rows);
   a.ws_loss = (float*)(ws + wl.off_loss);
   a.ws_flags = (uint8_t*)(ws + wl.off_flags);
   a.logp_out = logp_out;
@@ -493,8 +482,7 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
 // the workspace starts undefined).
 inline occ_status launch_k0(const K2Args& a, cudaStream_t s) {
   k0_count_valid<kK0Threads><<<1, kK0Threads, 0, s>>>(a.mask, a.ids, a.T, a.V,
-                                                      const_cast<long long*>(a.ws_N), a.ws_err,
-                                                      a.ws_rows);
+                                                      const_cast<long long*>(a.ws_N), a.ws_err);
   return check_launch("k0_count_valid");
 }
 

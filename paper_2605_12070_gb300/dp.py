@@ -44,7 +44,7 @@ def _allreduce_bits_or(word, group=None):
 
 def allreduce_loss_stats(stats, group=None):
     """In-place sum of loss_sum, loss and the four counters over ranks; the
-    err bits are OR-ed (a rank's BAD_ID and another's TIMEOUT both survive).
+    err bits are OR-ed (a bit set on any rank is set in the result).
     ``denom`` is left as is: every rank must have used the same global
     denominator."""
     if stats.dtype != torch.uint8 or stats.numel() != 64:

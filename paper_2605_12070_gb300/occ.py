@@ -26,7 +26,7 @@ LIB_PATH = os.path.join(_HERE, "libocc.so")
 OCC_OK = 0
 OCC_F32, OCC_BF16 = 0, 1
 FLAG_IN_BAND, FLAG_CLIPPED, FLAG_ACTIVE, FLAG_VALID = 1, 2, 4, 8
-DATA_ERR_BAD_ID, DATA_ERR_TIMEOUT = 1, 2
+DATA_ERR_BAD_ID = 1
 
 LOSS_STATS_BYTES = 64     # sizeof(occ_loss_stats)
 EWMA_STATE_BYTES = 40     # sizeof(occ_ewma_state)
@@ -42,8 +42,7 @@ EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_
 
 # occ_option codes (include/occ.h)
 OPTIONS = {"k1_warp": 0, "k1_threads": 1, "k2_threads": 2, "k2_head_bytes": 3, "k2_unroll": 4,
-           "fused_variant": 5, "fused_threads": 6, "fused_head_bytes": 7,
-           "test_lost_copy_row": 8, "test_wait_ns": 9}
+           "fused_threads": 5, "fused_head_bytes": 6}
 
 
 class OccError(RuntimeError):

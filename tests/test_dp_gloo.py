@@ -60,9 +60,9 @@ def _worker(rank, world, port, q):
         N = dp.global_token_count(n_local)
         lt, _ = oracle.token_logprob(z[rows], ids[rows])
         o = oracle.token_terms(lt, lo[rows], lmu[rows], adv[rows], mask[rows], p, N=N)
-        # rank 0 reports a dropped id, rank 1 a timed-out wait plus the sign bit:
+        # rank 0 reports a dropped id, rank 1 two other bits (one the sign bit):
         # the reduced word must keep every bit (OR), which MAX would not
-        err = occ.DATA_ERR_BAD_ID if rank == 0 else (occ.DATA_ERR_TIMEOUT | -2 ** 31)
+        err = occ.DATA_ERR_BAD_ID if rank == 0 else (2 | -2 ** 31)
         stats = _stats_bytes(o, N, err=err)
         dp.allreduce_loss_stats(stats)
         s = occ.decode_loss_stats(stats)
@@ -100,6 +100,6 @@ def test_sharded_batch_equals_unsharded():
             ref["n_valid"], ref["n_rd_out"], ref["n_clipped"], ref["n_active"])
         assert abs(s.loss - ref["loss"]) < 1e-12 and abs(s.loss_sum - ref["loss_sum"]) < 1e-12
         assert s.denom == ref["N"]
-        assert s.err == (occ.DATA_ERR_BAD_ID | occ.DATA_ERR_TIMEOUT | -2 ** 31)
+        assert s.err == (occ.DATA_ERR_BAD_ID | 2 | -2 ** 31)
         assert reset == ref_reset
     assert res[0][3] == res[1][3]

@@ -201,6 +201,6 @@ def test_options_are_explicit_and_checked(L):
     assert L.occ_set_option(2, 300) == 1 and L.occ_get_option(2) == 256
     assert L.occ_set_option(2, -1) == 0 and L.occ_get_option(2) == -1
     assert L.occ_set_option(99, 1) == 1 and L.occ_get_option(99) == -1
-    with occ.options(fused_variant=1, test_wait_ns=1000):
-        assert occ.get_option("fused_variant") == 1 and occ.get_option("test_wait_ns") == 1000
-    assert occ.get_option("fused_variant") == -1 and occ.get_option("test_wait_ns") == -1
+    with occ.options(fused_threads=256, fused_head_bytes=4096):
+        assert occ.get_option("fused_threads") == 256 and occ.get_option("fused_head_bytes") == 4096
+    assert occ.get_option("fused_threads") == -1 and occ.get_option("fused_head_bytes") == -1
