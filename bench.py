@@ -60,10 +60,11 @@ def parse_args():
     ap.add_argument("--loss-path", default="fused", choices=["fused", "two-call"],
                     help="fused: one launch reads old and current logits (occ_decoupled_loss_fused); "
                          "two-call: occ_token_logprob then occ_decoupled_loss_fwd_bwd")
-    ap.add_argument("--write-traffic", nargs=4, metavar=("CSV", "T", "N_VALID", "N_PARAMS"),
-                    help="no GPU: turn an ncu CSV of dram__bytes_{read,write}.sum (a run of this "
-                         "script on --workload with T tokens, N_VALID of them valid, and N_PARAMS "
-                         "EWMA parameters) into profiles/traffic_per_unit.json")
+    ap.add_argument("--write-traffic", nargs=4, metavar=("CSVS", "T", "N_VALID", "N_PARAMS"),
+                    help="no GPU: turn ncu CSVs of dram__bytes_{read,write}.sum (comma-separated, "
+                         "one capture per kernel, of a run of this script on --workload with T "
+                         "tokens, N_VALID of them valid, and N_PARAMS EWMA parameters) into "
+                         "profiles/traffic_per_unit.json")
     return ap.parse_args()
 
 
@@ -192,12 +193,15 @@ _TRAFFIC_KERNELS = {"k1_logprob_vec": "k1_token_logprob", "k2_loss_l2": "k2_deco
 
 
 def write_traffic(csv_path, workload, V, T, n_valid, n_params, command, path=TRAFFIC_JSON):
-    """Averages each kernel's DRAM bytes over its captured launches and stores
+    """Reads one or more ncu CSVs (comma-separated paths; one capture per
+    kernel), averages each kernel's DRAM bytes over its captured launches and stores
     them per unit (tokens, valid tokens, parameters) with the kernel's source
     hash in profiles/traffic_per_unit.json."""
     import csv
-    with open(csv_path) as f:
-        rows = list(csv.DictReader([ln for ln in f if ln.startswith('"')]))
+    rows = []
+    for one in csv_path.split(","):
+        with open(one) as f:
+            rows += list(csv.DictReader([ln for ln in f if ln.startswith('"')]))
     acc = {}
     for r in rows:
         name = r["Kernel Name"].split("(")[0].replace("void ", "").strip()
@@ -222,8 +226,9 @@ def write_traffic(csv_path, workload, V, T, n_valid, n_params, command, path=TRA
         e["source_hash"] = kernel_source_hash(key)
         kernels[key] = e
     out = {
-        "what": (f"DRAM bytes per unit from one ncu capture (dram__bytes_read.sum, "
-                 f"dram__bytes_write.sum) of a run with T={T} tokens ({n_valid} valid) and "
+        "what": (f"DRAM bytes per unit from ncu captures, one kernel per capture "
+                 f"(dram__bytes_read.sum, dram__bytes_write.sum), of a run with T={T} tokens "
+                 f"({n_valid} valid) and "
                  f"{n_params} EWMA parameters, averaged over the captured launches of each "
                  f"kernel; bench.py scales them to its workload by the units processed (valid "
                  f"tokens for the logits reads of the loss kernels, tokens for everything else, "
@@ -370,13 +375,18 @@ def cpu_baseline(batch, n_params_full, seconds):
 
 # ----------------------------------------------------------------- main
 
+# The small case the traffic captures run on, and the captures themselves:
+# one kernel per ncu run (an exact kernel name, two launches after the first),
+# each after the same command has exited 0 without ncu.
+TRAFFIC_CASE = ("python bench.py --tokens 4096 --ewma-n 200000000 --steps 2 --warmup 1 --no-e2e "
+                "--no-cpu-baseline --no-graph")
+TRAFFIC_KERNELS = ("k2_fused_l2", "k1_logprob_vec", "k2_loss_l2", "k3_ewma_vec")
 TRAFFIC_COMMAND = (
-    "python bench.py --tokens 4096 --ewma-n 400000000 --steps 2 --warmup 1 --no-e2e "
-    "--no-cpu-baseline --no-graph > plain_small.log && ncu --metrics dram__bytes_read.sum,"
-    "dram__bytes_write.sum,lts__t_sector_hit_rate.pct,gpu__time_duration.sum --clock-control none "
-    "-k regex:k[0-9]_ -c 40 --csv --log-file traffic_small.csv python bench.py --tokens 4096 "
-    "--ewma-n 400000000 --steps 2 --warmup 1 --no-e2e --no-cpu-baseline --no-graph; then "
-    "python bench.py --write-traffic traffic_small.csv 4096 <valid tokens> 400000000")
+    TRAFFIC_CASE + " > plain_small.log && for k in " + " ".join(TRAFFIC_KERNELS) + "; do "
+    "ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum "
+    "--clock-control none -k regex:^$k -s 1 -c 2 --csv --log-file traffic_$k.csv " + TRAFFIC_CASE +
+    " > /dev/null || break; done; then python bench.py --write-traffic "
+    + ",".join(f"traffic_{k}.csv" for k in TRAFFIC_KERNELS) + " 4096 <valid tokens> 200000000")
 
 
 def main():

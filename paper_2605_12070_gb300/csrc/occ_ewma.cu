@@ -191,14 +191,25 @@ __device__ __forceinline__ float load1(const bf16_t* p) {
 // eight parameters per vector, U vectors of each operand in flight per thread;
 // elements [8 n8, n) in a scalar tail.  On a copy step (b = 1) theta_prox is
 // not read.
-// Resident CTAs per SM: the launcher sizes the grid to one full wave of them.
+// Launch shape of the bf16 update (measured on GB300 over 4e9 parameters,
+// fraction of the measured copy bandwidth, float32 theta nearest / stochastic
+// and bf16 theta stochastic): 2 vectors of each operand in flight per thread
+// and grids of 6 / 8 CTAs of 256 threads per SM reach 1.05 / 1.03 and 0.97;
+// 4 vectors in flight with one resident wave of 3 / 4 CTAs per SM reached
+// 0.95 / 0.93 and 0.94, 1 vector 0.98 / 0.97 and 0.84, 512-thread CTAs 0.89 /
+// 0.86 and 0.90.  The register bound keeps 3 / 4 CTAs resident at least.
+constexpr int kK3Bf16Unroll = 2;
 template <typename ThT>
-constexpr int k3_bf16_ctas_per_sm() {
+constexpr int k3_bf16_min_ctas() {
   return sizeof(ThT) == 4 ? 3 : 4;
+}
+template <typename ThT>
+constexpr int k3_bf16_grid_per_sm() {
+  return sizeof(ThT) == 4 ? 6 : 8;
 }
 
 template <typename ThT, int NT, int U>
-__global__ void __launch_bounds__(NT, k3_bf16_ctas_per_sm<ThT>())
+__global__ void __launch_bounds__(NT, k3_bf16_min_ctas<ThT>())
     k3_ewma_bf16(bf16_t* __restrict__ tp, const ThT* __restrict__ th, int64_t n, bool vec,
                  const occ_ewma_state* __restrict__ st, uint64_t seed, uint64_t idx0) {
   const double bd = st->coef_b;
@@ -321,18 +332,18 @@ occ_status launch_bf16_body(bf16_t* tp, const void* th, occ_dtype theta_dt, int6
   if (n == 0) return OCC_OK;
   const bool vec = aligned(tp, 16) && aligned(th, 16);
   const int64_t work = vec ? (n + 7) / 8 : n;
-  const int64_t need = (work + kK3Threads * kK3Unroll - 1) / (kK3Threads * kK3Unroll);
+  const int64_t need = (work + kK3Threads * kK3Bf16Unroll - 1) / (kK3Threads * kK3Bf16Unroll);
   auto grid_for = [&](int per_sm) {
     return (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, (int64_t)sm_count() * per_sm));
   };
   note_kernel("k3_ewma_bf16");
   if (theta_dt == OCC_BF16)
-    k3_ewma_bf16<bf16_t, kK3Threads, kK3Unroll>
-        <<<grid_for(k3_bf16_ctas_per_sm<bf16_t>()), kK3Threads, 0, s>>>(tp, (const bf16_t*)th, n,
+    k3_ewma_bf16<bf16_t, kK3Threads, kK3Bf16Unroll>
+        <<<grid_for(k3_bf16_grid_per_sm<bf16_t>()), kK3Threads, 0, s>>>(tp, (const bf16_t*)th, n,
                                                                          vec, st, seed, idx0);
   else
-    k3_ewma_bf16<float, kK3Threads, kK3Unroll>
-        <<<grid_for(k3_bf16_ctas_per_sm<float>()), kK3Threads, 0, s>>>(tp, (const float*)th, n,
+    k3_ewma_bf16<float, kK3Threads, kK3Bf16Unroll>
+        <<<grid_for(k3_bf16_grid_per_sm<float>()), kK3Threads, 0, s>>>(tp, (const float*)th, n,
                                                                         vec, st, seed, idx0);
   return check_launch("k3_ewma_bf16");
 }
