@@ -89,10 +89,11 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
     acc_init(acc);
     // Row walk (GB300, bf16, against one load at a time in the last round):
     // clamped rounds in the 128- and 512-thread tiers (V = 151936: 6.31 -> 5.93
-    // ms; 32000: 1.48 -> 1.37 ms; 24000: 1.34 -> 1.18 ms), one load at a time
-    // in the 256-thread tier (V = 50000: 1.30 against 1.33 ms) and for peeled
-    // rows (V = 50257: 1.32 against 1.35 ms).
-    constexpr Walk kW = (PEEL || NT == 256) ? Walk::kSerialTail : Walk::kClampAll;
+    // ms; 32000: 1.48 -> 1.37 ms; 24000: 1.34 -> 1.18 ms; peeled 32001: 1.64 ->
+    // 1.47 ms), one load at a time in the 256-thread tier (V = 50000: 1.30
+    // against 1.33 ms) and for peeled rows of the larger tiers (V = 50257: 1.32
+    // against 1.35 ms).
+    constexpr Walk kW = (NT == 256 || (PEEL && NT != 128)) ? Walk::kSerialTail : Walk::kClampAll;
     const int nh = (int)head;
     walk_row<kW, U, NT>(
         tid, (int)nvec, [&](int j) { return ld_hint_v4(zv + j, keep); },
