@@ -12,10 +12,13 @@ the token-mean loss (1e-4 relative; Eqs. 2-4).  dlogits (R8) are compared in
 chunks on more than 2048 rows drawn from every token class: active, clipped,
 out of band, masked, and rows of every class at the batch edges.
 
-The last test chains the 7.6e9-parameter float32 EWMA update (App. B, with
-the auto-reset of Sec. 5.2) on the device statistics of that loss step and
-checks rho, the reset decision, the state and about 3 M sampled parameters
-against the oracle, whose own reset decision comes from its own counters.
+The interpolation proxies of Table 1 (log pi_old built per token inside K2)
+and the per-token entropy / KL diagnostics of the fused pass are compared on
+every token of the same batch too.  The last test chains the 7.6e9-parameter
+float32 EWMA update (App. B, with the auto-reset of Sec. 5.2) on the device
+statistics of that loss step and checks rho, the reset decision, the state and
+about 3 M sampled parameters against the oracle, whose own reset decision
+comes from its own counters.
 """
 
 import numpy as np
@@ -252,3 +255,50 @@ def test_ewma_7p6e9_chained_on_the_loss_statistics(agentic):
         th.add_(1e-4)   # the next actor parameters
     # the ragged end of the buffer was covered
     assert idx[-1] == n - 1
+
+
+@pytest.mark.parametrize("kind,alpha", [("loglinear", 0.5), ("arithmetic", 1.0 / 3.0)])
+def test_proxies_every_token(agentic, kind, alpha):
+    """F2 on the full batch: log pi_old is built per token from mu_old and
+    pi_theta (Table 1, App. A) inside K2; a band of [0.95, 1.05] puts tokens
+    on both sides of it.  Every token against the oracle; dlogits on rows of
+    every class."""
+    b, _, lt64, lse = agentic
+    p = dict(b.thresholds(), rd_lo=0.95, rd_hi=1.05)
+    lp_prox = orc.proxy_logprob(kind, alpha, b.logp_mu.cpu().numpy(), np.nan_to_num(lt64))
+    params = loss_params(b, rd_lo=0.95, rd_hi=1.05)
+    o = oracle_loss(b, lt64, lp_prox, params)
+    out = occ.occ_decoupled_loss_fwd_bwd(b.z_theta, b.ids, None, b.logp_mu, b.adv, b.mask,
+                                         proxy=kind, alpha=alpha, **p)
+    torch.cuda.synchronize()
+    st, gfl = _check_every_token(b, out, o, lt64, None, None)
+    assert 0 < st.n_rd_out < st.n_valid and 0 < st.n_active
+    rows, _ = _dz_rows(o, gfl, b.T, np.random.default_rng(14),
+                       ("active", "out_of_band", "masked"), per_class=700)
+    _check_dlogits(b, out["dlogits"], o, lse, rows)
+
+
+def test_diagnostics_every_token(agentic):
+    """F3 on the full batch: per-token entropy of pi_theta and KL(pi_old ||
+    pi_theta) from the fused pass, every valid token against the textbook
+    definitions (float32 weighted sums of O(10) logits: 1e-4 absolute)."""
+    b = agentic[0]
+    out = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                       dlogits=None, want_diagnostics=True, **b.thresholds())
+    torch.cuda.synchronize()
+
+    def fn(r):
+        it = torch.as_tensor(r, device="cuda")
+        z = to_f64(b.z_theta[it])
+        zo = to_f64(b.z_old[it])
+        return orc.token_entropy(z), orc.token_kl(zo, z)
+
+    parts = map_row_chunks(fn, np.arange(b.T), chunk=64)
+    H = np.concatenate([p[0] for p in parts])
+    K = np.concatenate([p[1] for p in parts])
+    valid = b.mask.cpu().numpy() != 0
+    gh = out["entropy"].cpu().numpy().astype(np.float64)
+    gk = out["kl"].cpu().numpy().astype(np.float64)
+    assert np.abs(gh[valid] - H[valid]).max() <= 1e-4
+    assert np.abs(gk[valid] - K[valid]).max() <= 1e-4
+    assert np.all(gh[~valid] == 0.0) and np.all(gk[~valid] == 0.0)
