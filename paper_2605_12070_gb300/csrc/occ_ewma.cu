@@ -220,25 +220,45 @@ __global__ void __launch_bounds__(NT, k3_bf16_min_ctas<ThT>())
   int64_t done = 0;
   if (vec) {
     const int64_t n8 = n / 8;
+    // The rounding is written to keep the integer (ALU) pipe light, which
+    // otherwise co-limits the bf16-theta update: nearest-even rounds a pair per
+    // conversion; the stochastic path checks the eight values for inf / NaN
+    // once, with multiplies (0 * v is NaN only for them), takes each 16-bit
+    // lane of the generator outputs in one operation, and packs two rounded
+    // values with one byte permutation.  The bits are those of
+    // round_bf16_bits, which the rare vector holding inf or NaN still takes.
     auto emit = [&](int64_t iv, const uint4& xr, const Raw8<ThT>& yr) {
-      float x[8], y[8];
+      float x[8], y[8], v[8];
       Elem<bf16_t>::unpack(xr, x);
       yr.unpack(y);
-      uint16_t o[8];
-      const uint64_t g0 = idx0 + 8 * iv;  // idx0 is a multiple of 8: two whole generator outputs
-      uint64_t r0 = 0, r1 = 0;
-      if (seed) {
-        r0 = splitmix64_at(seed, g0 >> 2);
-        r1 = splitmix64_at(seed, (g0 >> 2) + 1);
-      }
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const float v = copy ? y[k] : fmaf(b, y[k] - x[k], x[k]);
-        const uint64_t r = k < 4 ? r0 : r1;
-        o[k] = round_bf16_bits(v, seed != 0, (uint32_t)(r >> (16 * (k & 3))) & 0xffffu);
+      for (int k = 0; k < 8; ++k) v[k] = copy ? y[k] : fmaf(b, y[k] - x[k], x[k]);
+      uint32_t w[4];
+      if (!seed) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) w[j] = pack_bf16x2(v[2 * j], v[2 * j + 1]);
+      } else {
+        const uint64_t g0 = idx0 + 8 * iv;  // idx0 is a multiple of 8: two whole generator outputs
+        const uint64_t r0 = splitmix64_at(seed, g0 >> 2);
+        const uint64_t r1 = splitmix64_at(seed, (g0 >> 2) + 1);
+        const uint32_t q[4] = {(uint32_t)r0, (uint32_t)(r0 >> 32), (uint32_t)r1,
+                               (uint32_t)(r1 >> 32)};
+        float s = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) s = fmaf(v[k], 0.f, s);
+        if (s == 0.f) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)  // lanes 2j, 2j + 1 = low and high half of q[j]
+            w[j] = __byte_perm(__float_as_uint(v[2 * j]) + (q[j] & 0xffffu),
+                               __float_as_uint(v[2 * j + 1]) + (q[j] >> 16), 0x7632);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            w[j] = (uint32_t)round_bf16_bits(v[2 * j], true, q[j] & 0xffffu) |
+                   ((uint32_t)round_bf16_bits(v[2 * j + 1], true, q[j] >> 16) << 16);
+        }
       }
-      st_stream_v4(tp + 8 * iv, make_uint4(o[0] | ((uint32_t)o[1] << 16), o[2] | ((uint32_t)o[3] << 16),
-                                           o[4] | ((uint32_t)o[5] << 16), o[6] | ((uint32_t)o[7] << 16)));
+      st_stream_v4(tp + 8 * iv, make_uint4(w[0], w[1], w[2], w[3]));
     };
     int64_t i = gtid;
     for (; i + (int64_t)(U - 1) * stride < n8; i += (int64_t)U * stride) {
