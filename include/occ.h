@@ -347,12 +347,12 @@ occ_status occ_host_alloc(size_t bytes, void** out);
 occ_status occ_host_free(void* ptr, size_t bytes);
 
 /*
- * occ_set_option / occ_get_option -- tuning and test controls.  (The paper
- * has no counterpart: these are measurement plumbing.)
+ * occ_set_option / occ_get_option -- launch-shape overrides.  (The paper has
+ * no counterpart: these are measurement plumbing.)
  *
- * Every call picks its kernel and launch shape by itself; an option overrides
- * that choice, for measurements (sweeps of CTA sizes and shared-memory heads,
- * measurements of the launch shapes.
+ * Every call picks its kernel's launch shape by itself; an option overrides
+ * that choice for measurements (sweeps of CTA sizes, shared-memory heads and
+ * loads in flight).  Every shape meets the same accuracy bounds.
  * The library reads no environment variable: an option changes only when a
  * caller sets it.  Options are process-wide and read when a call is launched;
  * set them between calls.  A value of -1 restores the automatic choice.

@@ -130,7 +130,7 @@ def lib():
 
 
 def set_option(name, value):
-    """Sets a process-wide tuning or test option (-1 = automatic / off)."""
+    """Sets a process-wide launch-shape option (-1 = automatic)."""
     _check(lib().occ_set_option(OPTIONS[name], int(value)), f"occ_set_option({name})")
 
 
