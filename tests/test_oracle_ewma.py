@@ -156,6 +156,15 @@ def test_fma_f32_single_rounding():
     c[:8] = np.float32(1.0)
     a[:8] = np.float32(2.0 ** -24)
     b[:8] = np.float32(1.0) + np.float32(2.0 ** -23) * np.arange(8, dtype=np.float32)
+    # a*b = (1 + 2^-12)^2 = 1 + 2^-11 + 2^-24 is exactly a float32 midpoint, and a
+    # tiny c (below float64 resolution at 1) makes the float64 sum land on it while
+    # the exact value lies just above or below: only the sum's rounding error tells
+    # which way to round (both signs, several scales)
+    k = np.arange(8, 16)
+    scale = np.float32(2.0) ** ((k % 4) - 2).astype(np.float32)
+    a[8:16] = (np.float32(1.0) + np.float32(2.0 ** -12)) * scale
+    b[8:16] = np.float32(1.0) + np.float32(2.0 ** -12)
+    c[8:16] = np.where(k % 2 == 0, 1.0, -1.0).astype(np.float32) * np.float32(2.0 ** -60) * scale
     got = fma_f32(a, b, c)
     for i in range(2000):
         exact = Fraction(float(a[i])) * Fraction(float(b[i])) + Fraction(float(c[i]))

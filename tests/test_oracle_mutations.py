@@ -71,6 +71,16 @@ MUTATIONS = [
      "arithmetic proxy weights transposed"),
     ("diagnostics.py", "return (np.exp(lq) * (lq - lp)).sum(axis=1)",
      "return (np.exp(lp) * (lq - lp)).sum(axis=1)", "KL weighted by the wrong distribution"),
+    ("diagnostics.py", "return -(np.exp(lp) * lp).sum(axis=1)",
+     "return (np.exp(lp) * lp).sum(axis=1)", "entropy sign"),
+    ("ewma.py", "b = 1.0 / w", "b = 1.0 / (w + 1.0)", "new-parameter weight off by one"),
+    ("ewma.py", "new = th.copy() if reset else a * tp + b * th",
+     "new = tp.copy() if reset else a * tp + b * th", "a reset keeps the old proximal parameters"),
+    ("ewma.py", "out = ((u + r) >> np.uint64(16)) & np.uint64(0xFFFF)",
+     "out = ((u + r + np.uint64(0x8000)) >> np.uint64(16)) & np.uint64(0xFFFF)",
+     "rounding offset added on top of the random bits"),
+    ("ewma.py", "fix = (np.abs(d) == half) & (d * e > 0)",
+     "fix = (np.abs(d) == half) & (d * e < 0)", "float32 FMA midpoint resolved the wrong way"),
 ]
 
 
