@@ -122,17 +122,21 @@ def sr_bits(seed, idx):
 def round_bf16(x32, seed=0, idx=None):
     """float32 -> bf16 bits.  seed == 0: nearest, ties to even.  Otherwise add 16
     random bits (``sr_bits``) below the bf16 unit in the last place and
-    truncate (stochastic rounding of the magnitude)."""
+    truncate (stochastic rounding of the magnitude).  Infinities are exact; a
+    NaN rounds to a quiet NaN of the same sign (0x7FC0 with the sign bit), as
+    rounding must keep a NaN a NaN whatever bits its payload holds."""
     u = np.asarray(x32, dtype=np.float32).view(np.uint32).astype(np.uint64)
     special = (u & np.uint64(0x7F800000)) == np.uint64(0x7F800000)
+    nan = special & ((u & np.uint64(0x007FFFFF)) != np.uint64(0))
     if seed == 0:
         lsb = (u >> np.uint64(16)) & np.uint64(1)
         r = np.uint64(0x7FFF) + lsb
     else:
         r = sr_bits(seed, idx)
     out = ((u + r) >> np.uint64(16)) & np.uint64(0xFFFF)
-    trunc = (u >> np.uint64(16)) & np.uint64(0xFFFF)
-    return np.where(special, trunc, out).astype(np.uint16)
+    trunc = (u >> np.uint64(16)) & np.uint64(0xFFFF)          # exact for the infinities
+    quiet = ((u >> np.uint64(16)) & np.uint64(0x8000)) | np.uint64(0x7FC0)
+    return np.where(nan, quiet, np.where(special, trunc, out)).astype(np.uint16)
 
 
 def fma_f32(a, b, c):
@@ -142,16 +146,20 @@ def fma_f32(a, b, c):
     exact up to its TwoSum error e.  Rounding s = fl64(p + c) to float32 is
     then correct except when s falls exactly on a float32 midpoint, where the
     sign of e decides the side."""
-    p = np.asarray(a, np.float64) * np.asarray(b, np.float64)
-    c = np.asarray(c, np.float64)
-    s = p + c
-    bp = s - p
-    e = (p - (s - bp)) + (c - bp)                  # TwoSum: p + c = s + e exactly
-    r = s.astype(np.float32)
-    d = s - r.astype(np.float64)                   # exact
-    half = np.spacing(np.abs(r)).astype(np.float64) / 2
-    fix = (np.abs(d) == half) & (d * e > 0)        # past the midpoint: round away from r
-    r = np.where(fix, np.nextafter(r, np.where(d > 0, np.float32(np.inf), np.float32(-np.inf))), r)
+    # (for an infinite or NaN operand the TwoSum terms are NaN, the midpoint test
+    # is false and r is the float32 of s: inf or NaN, as a fused multiply-add gives)
+    with np.errstate(invalid="ignore"):
+        p = np.asarray(a, np.float64) * np.asarray(b, np.float64)
+        c = np.asarray(c, np.float64)
+        s = p + c
+        bp = s - p
+        e = (p - (s - bp)) + (c - bp)              # TwoSum: p + c = s + e exactly
+        r = s.astype(np.float32)
+        d = s - r.astype(np.float64)               # exact
+        half = np.spacing(np.abs(r)).astype(np.float64) / 2
+        fix = (np.abs(d) == half) & (d * e > 0)    # past the midpoint: round away from r
+        r = np.where(fix, np.nextafter(r, np.where(d > 0, np.float32(np.inf), np.float32(-np.inf))),
+                     r)
     return r.astype(np.float32)
 
 
@@ -161,6 +169,7 @@ def ewma_update_bf16(tp_bits, theta32, b, copy, seed=0, idx0=0):
     step), rounded to bf16."""
     tp = bf16_bits_to_f32(tp_bits)
     th = np.asarray(theta32, dtype=np.float32)
-    v = th if copy else fma_f32(np.float32(b), (th - tp).astype(np.float32), tp)
+    with np.errstate(invalid="ignore"):            # signalling-NaN parameters stay NaN
+        v = th if copy else fma_f32(np.float32(b), (th - tp).astype(np.float32), tp)
     idx = np.arange(idx0, idx0 + tp.size, dtype=np.uint64)
     return round_bf16(v, seed, idx)

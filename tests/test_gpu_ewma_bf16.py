@@ -45,6 +45,38 @@ def test_bf16_buffer_matches_oracle_bits(theta_dtype, seed, n, offset):
         th.add_(torch.full_like(th, 1e-3))
 
 
+@pytest.mark.parametrize("seed", [0, 12345])
+def test_infinities_and_nans_survive_the_update(seed):
+    # Non-finite parameters stay non-finite: inf stays inf, NaN stays NaN (all
+    # payloads, including one whose low bits alone are set and one with every
+    # mantissa bit set), and their finite neighbours in the same 8-parameter
+    # vector round exactly as the oracle does.
+    n = 4096
+    th32, tp32 = make_ewma_buffers(n, seed=9, device="cuda")
+    special = {3: 0x7F800000, 10: 0xFF800000, 17: 0x7FC00000, 24: 0x7FFFFFFF, 31: 0x7F800001,
+               40: 0xFFFFFFFF, 1000: 0x7F800000, 4095: 0x7FC00001}
+    raw = th32.view(torch.int32)
+    for i, b in special.items():
+        raw[i] = b - (1 << 32) if b >= 1 << 31 else b
+    tp = tp32.to(torch.bfloat16)
+    before = _bits(tp)
+    st = occ.new_ewma_state("cuda", w0=3.0)
+    occ.occ_ewma_update_bf16(tp, th32, 0.75, st, sr_seed=seed)
+    torch.cuda.synchronize()
+    a, b, reset, _ = oracle.ewma_coefficients(oracle.EwmaState(w=3.0), 0.75)
+    ref = oracle.ewma_update_bf16(before, th32.cpu().numpy(), np.float32(b), reset, seed=seed)
+    got = _bits(tp)
+    idx = np.array(sorted(special))
+    finite = np.ones(n, dtype=bool)
+    finite[idx] = False
+    assert np.array_equal(got[finite], ref[finite])
+    x = th32.cpu().numpy()[idx]
+    assert np.all((got[idx] & 0x7F80) == 0x7F80)                     # still non-finite
+    assert np.all(((got[idx] & 0x7F) != 0) == np.isnan(x))          # NaN iff NaN
+    inf = np.isinf(x)
+    assert np.array_equal(got[idx][inf], ref[idx][inf])              # infinities exact
+
+
 def test_bf16_reset_copies_bf16_theta_exactly():
     th32, tp32 = make_ewma_buffers(100_000, seed=1, device="cuda")
     th = th32.to(torch.bfloat16)

@@ -174,3 +174,25 @@ def test_fma_f32_single_rounding():
         best = min(cands, key=lambda x: (abs(Fraction(float(x)) - exact),
                                         int(np.float32(x).view(np.uint32)) & 1))
         assert got[i] == best, i
+
+
+def test_bf16_rounding_keeps_infinities_and_nans():
+    # inf stays inf and NaN stays NaN (sign kept) under both roundings, whatever
+    # the payload: adding the rounding increment to a NaN whose mantissa bits are
+    # all set would carry into the sign bit and give a zero.  Finite values at the
+    # top of the range round to the largest bf16 or to inf as float32 -> bf16
+    # rounding to nearest does (torch's conversion).
+    torch = pytest.importorskip("torch")
+    from oracle import round_bf16
+    bits = np.array([0x7F800000, 0xFF800000, 0x7FC00000, 0x7FFFFFFF, 0xFFFFFFFF, 0x7F800001,
+                     0xFFC00001], dtype=np.uint32)
+    x = bits.view(np.float32)
+    for seed in (0, 1, 77, 2 ** 40 + 3):
+        out = round_bf16(x, seed, np.arange(x.size, dtype=np.uint64))
+        exp_all_ones = (out & 0x7F80) == 0x7F80
+        assert np.all(exp_all_ones), (seed, [hex(v) for v in out])
+        assert np.all((out & 0x8000) == ((bits >> 16) & 0x8000)), seed      # sign kept
+        assert np.all(((out & 0x7F) != 0) == np.isnan(x)), seed              # NaN iff NaN
+    big = np.array([3.3895e38, 3.39e38, 3.4e38, -3.4e38], dtype=np.float32)
+    want = torch.from_numpy(big).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(round_bf16(big, 0), want)

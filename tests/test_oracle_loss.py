@@ -361,3 +361,22 @@ def test_open_band_role_weights_by_the_total_ratio():
                                                   eps_high=1e9, rd_weight=0))
     expect0 = -math.fsum(np.exp(lt[v] - lo[v]) * A[v]) / v.sum()
     assert abs(o0["loss"] - expect0) <= 1e-12 * max(1.0, abs(expect0))
+
+
+def test_threshold_distances_measure_to_the_deciding_edge():
+    # The exemption from bit-exactness is decided by the distance, in log-ratio
+    # space, to the threshold that decides the token: the clip edge of the
+    # advantage's sign (log(1 + eps_high) for A >= 0, log(1 - eps_low) for A < 0)
+    # and the nearer band edge.  Hand-built tokens at known distances.
+    p = LossParams(0.5, 2.0, 0.2, 0.28)
+    d = np.array([1e-7, -3e-7, 2e-3, -5e-4])
+    edge_hi, edge_lo = np.log1p(0.28), np.log1p(-0.2)
+    for A, edge in ((1.0, edge_hi), (0.0, edge_hi), (-1.0, edge_lo)):
+        lt = edge + d                       # log pi_theta, with log pi_old = 0
+        o = token_terms(lt, np.zeros(4), np.zeros(4), np.full(4, A), None, p)
+        assert np.allclose(o["dist_rs"], np.abs(d), rtol=0, atol=1e-12), A
+        assert np.allclose(o["dist_rd"], np.log(2.0), rtol=0, atol=1e-12)   # log r_d = 0
+    for edge in (np.log(0.5), np.log(2.0)):
+        lo_ = edge + d                      # log pi_old, with log mu_old = 0
+        o = token_terms(lo_, lo_, np.zeros(4), np.ones(4), None, p)
+        assert np.allclose(o["dist_rd"], np.abs(d), rtol=0, atol=1e-12), edge

@@ -81,6 +81,25 @@ MUTATIONS = [
      "rounding offset added on top of the random bits"),
     ("ewma.py", "fix = (np.abs(d) == half) & (d * e > 0)",
      "fix = (np.abs(d) == half) & (d * e < 0)", "float32 FMA midpoint resolved the wrong way"),
+    ("loss.py", "flags = (in_band * FLAG_IN_BAND + (~mis) * FLAG_CLIPPED",
+     "flags = (in_band * FLAG_IN_BAND + mis * FLAG_CLIPPED", "clip flag inverted"),
+    ("loss.py", "n_rd_out=int(np.sum(valid & ~in_band))", "n_rd_out=int(np.sum(~in_band))",
+     "out-of-band count includes masked tokens"),
+    ("loss.py", "    ok = (ids >= 0) & (ids < V)\n", "    ok = (ids >= 0) & (ids <= V + 1)\n",
+     "token ids past the vocabulary accepted"),
+    ("ewma.py", "n_valid > 0 and streak >= min_streak", "n_valid > 0 and streak > min_streak",
+     "reset one low step late"),
+    ("ewma.py", "EwmaState(w=1.0, streak=0, n_resets=state.n_resets + 1)",
+     "EwmaState(w=0.0, streak=0, n_resets=state.n_resets + 1)", "a reset empties the history weight"),
+    ("diagnostics.py", "return z - (M + np.log(np.exp(z - M).sum(axis=1, keepdims=True)))",
+     "return z - np.log(np.exp(z - M).sum(axis=1, keepdims=True))", "log-softmax without its shift"),
+    ("ewma.py", "np.where(nan, quiet, np.where(special, trunc, out))", "out",
+     "inf and NaN rounded like finite values"),
+    ("ewma.py", "np.where(nan, quiet, np.where(special, trunc, out))", "np.where(special, trunc, out)",
+     "NaN truncated (a low payload becomes inf)"),
+    ("loss.py", "dist_rs = np.where(A >= 0, np.abs(log_rs - np.log1p(p.eps_high))",
+     "dist_rs = np.where(A >= 0, np.abs(log_rs - np.log1p(p.eps_low))",
+     "clip-distance measured to the wrong edge"),
 ]
 
 
