@@ -380,3 +380,16 @@ def test_threshold_distances_measure_to_the_deciding_edge():
         lo_ = edge + d                      # log pi_old, with log mu_old = 0
         o = token_terms(lo_, lo_, np.zeros(4), np.ones(4), None, p)
         assert np.allclose(o["dist_rd"], np.abs(d), rtol=0, atol=1e-12), edge
+
+
+def test_bad_ids_are_counted_among_unmasked_tokens_only():
+    # Interface convention: a token whose id is outside [0, V) is dropped, and it
+    # counts as a bad id only if the loss mask keeps it (a masked token carries
+    # no evidence either way).
+    z = np.zeros((4, 5))
+    ids = np.array([1, 7, -1, 2])
+    mask = np.array([1, 1, 0, 1], dtype=np.uint8)
+    lt, _ = token_logprob(z, ids)
+    o = token_terms(lt, lt, lt, np.ones(4), mask, LossParams(0.5, 2.0, 0.2, 0.28),
+                    id_ok=(ids >= 0) & (ids < 5))
+    assert o["bad_ids"] == 1 and o["n_valid"] == 2 and o["N"] == 2

@@ -97,6 +97,11 @@ MUTATIONS = [
      "inf and NaN rounded like finite values"),
     ("ewma.py", "np.where(nan, quiet, np.where(special, trunc, out))", "np.where(special, trunc, out)",
      "NaN truncated (a low payload becomes inf)"),
+    ("loss.py", "bad_ids = int(np.sum(m & ~ok))", "bad_ids = int(np.sum(~ok))",
+     "masked tokens counted as bad ids"),
+    ("loss.py", "loss = loss_sum / N if N > 0 else 0.0", "loss = loss_sum / N if N > 0 else np.nan",
+     "empty batch gives NaN"),
+    ("loss.py", "    valid = m & ok\n", "    valid = m\n", "bad ids kept as valid tokens"),
     ("loss.py", "dist_rs = np.where(A >= 0, np.abs(log_rs - np.log1p(p.eps_high))",
      "dist_rs = np.where(A >= 0, np.abs(log_rs - np.log1p(p.eps_low))",
      "clip-distance measured to the wrong edge"),
