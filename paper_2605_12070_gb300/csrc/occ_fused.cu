@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
         };
         const int64_t nre = nvec - head;
         const uint4* zr = zv + head;
-        walk_row<kW, 2 * U, NT>(
+        walk_row<kW, 8, NT>(  // 8 vectors in flight, whatever the forward pass's U
             tid, (int)nre, [&](int j) { return ld_hint_v4(zr + j, last); },
             [&](int j, const uint4& r) { emit(head + j, r); });
 #pragma unroll 4
@@ -239,11 +239,16 @@ constexpr int kFusedUnroll = 4;
 
 using FusedKern = void (*)(const FusedArgs);
 
+// The diagnostics need two more accumulators and the per-element differences;
+// 3 row pairs in flight per thread keep that instantiation free of spills.
+constexpr int kFusedUnrollDiag = 3;
+
 template <typename Tin, typename Tout, bool DIAG, bool PEEL>
 static FusedKern fused_kernel(int nt) {
-  return nt == 128   ? k2_fused_l2<Tin, Tout, 128, kFusedUnroll, DIAG, PEEL>
-         : nt == 256 ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, DIAG, PEEL>
-                     : k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, DIAG, PEEL>;
+  constexpr int U = DIAG ? kFusedUnrollDiag : kFusedUnroll;
+  return nt == 128   ? k2_fused_l2<Tin, Tout, 128, U, DIAG, PEEL>
+         : nt == 256 ? k2_fused_l2<Tin, Tout, 256, U, DIAG, PEEL>
+                     : k2_fused_l2<Tin, Tout, kFusedThreads, U, DIAG, PEEL>;
 }
 
 // Rows off a 16-byte boundary run the vector kernel peeled when the old-logits
