@@ -225,6 +225,18 @@ def write_traffic(csv_path, workload, V, T, n_valid, n_params, command, path=TRA
         e["launches"] = len(d["dram__bytes_read.sum"])
         e["source_hash"] = kernel_source_hash(key)
         kernels[key] = e
+    # entries of kernels left out of this capture stay while their code is unchanged
+    try:
+        with open(path) as f:
+            old = json.load(f)
+        if old.get("workload") == workload and old.get("V") == V:
+            for key, e in old.get("kernels", {}).items():
+                if key not in kernels and key in KERNEL_SOURCES \
+                        and e.get("source_hash") == kernel_source_hash(key):
+                    kernels[key] = e
+    except (OSError, ValueError):
+        pass
+    kernels = dict(sorted(kernels.items()))
     out = {
         "what": (f"DRAM bytes per unit from ncu captures, one kernel per capture "
                  f"(dram__bytes_read.sum, dram__bytes_write.sum), of a run with T={T} tokens "

@@ -364,7 +364,7 @@ typedef enum {
   OCC_OPT_K1_THREADS = 1,      /* threads per occ_token_logprob CTA: 128, 256, 512   */
   OCC_OPT_K2_THREADS = 2,      /* threads per occ_decoupled_loss_fwd_bwd CTA: 128, 256, 512 */
   OCC_OPT_K2_HEAD_BYTES = 3,   /* its shared-memory head, bytes (0 = re-read all from L2) */
-  OCC_OPT_K2_UNROLL = 4,       /* vectors in flight per thread of its 512-thread kernel: 4, 8 */
+  OCC_OPT_K2_UNROLL = 4,       /* vectors in flight per thread of its 512-thread kernel: 4, 6, 8 */
   OCC_OPT_FUSED_THREADS = 5,   /* threads per occ_decoupled_loss_fused CTA: 128, 256, 512 */
   OCC_OPT_FUSED_HEAD_BYTES = 6, /* its shared-memory head, bytes                       */
   OCC_OPT_COUNT_ = 7

@@ -54,7 +54,7 @@ static bool option_value_ok(occ_option opt, int64_t v) {
     case OCC_OPT_K1_THREADS:
     case OCC_OPT_K2_THREADS:
     case OCC_OPT_FUSED_THREADS: return v == 128 || v == 256 || v == 512;
-    case OCC_OPT_K2_UNROLL: return v == 4 || v == 8;
+    case OCC_OPT_K2_UNROLL: return v == 4 || v == 6 || v == 8;
     case OCC_OPT_K2_HEAD_BYTES:
     case OCC_OPT_FUSED_HEAD_BYTES: return v >= 0 && v <= 227 * 1024 && v % 16 == 0;
     default: return false;

@@ -251,12 +251,17 @@ __global__ void __launch_bounds__(NT) k2_loss_stream(const K2Args a) {
 
 using K2Kern = void (*)(const K2Args);
 
+// Vectors in flight per thread of the 512-thread tier: 8 for aligned rows, 6
+// for peeled ones (V = 151937, GB300: 6.41 ms against 6.77 with 8, which
+// spills, and 6.55 with 4); `unroll` > 0 overrides.
 template <typename Tin, typename Tout, bool PEEL>
 static K2Kern l2_kernel(int nt, int unroll) {
-  return (nt == 128)     ? k2_loss_l2<Tin, Tout, 128, 8, PEEL>
-         : (nt == 256)   ? k2_loss_l2<Tin, Tout, 256, 8, PEEL>
-         : (unroll == 4) ? k2_loss_l2<Tin, Tout, 512, 4, PEEL>
-                         : k2_loss_l2<Tin, Tout, 512, 8, PEEL>;
+  const int u = unroll > 0 ? unroll : (PEEL ? 6 : 8);
+  return (nt == 128)   ? k2_loss_l2<Tin, Tout, 128, 8, PEEL>
+         : (nt == 256) ? k2_loss_l2<Tin, Tout, 256, 8, PEEL>
+         : (u == 4)    ? k2_loss_l2<Tin, Tout, 512, 4, PEEL>
+         : (u == 6)    ? k2_loss_l2<Tin, Tout, 512, 6, PEEL>
+                       : k2_loss_l2<Tin, Tout, 512, 8, PEEL>;
 }
 
 // Rows that are not 16-byte aligned can run the vector kernel peeled when the
@@ -288,7 +293,7 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     const int nt_auto = row_bytes <= 64 * 1024 ? 128 : row_bytes <= 112 * 1024 ? 256 : 512;
     const int64_t nt_opt = option(OCC_OPT_K2_THREADS);
     const int64_t head_opt = option(OCC_OPT_K2_HEAD_BYTES);
-    const int unroll = option(OCC_OPT_K2_UNROLL) == 4 ? 4 : 8;
+    const int unroll = (int)option(OCC_OPT_K2_UNROLL);  // -1: by the row layout
     const int nt = nt_opt > 0 ? (int)nt_opt : nt_auto;
     K2Kern kern = l2_kernel<Tin, Tout, false>(nt, unroll);
     if constexpr (sizeof(Tin) == sizeof(Tout))

@@ -49,3 +49,43 @@ def test_k2_launch_shape_against_oracle(shape, name, T, f32):
     g = np.abs(o["g"][pick])[:, None]
     rel = 2e-6 if f32 else 2.0 ** -8
     assert np.all(np.abs(got - ref) <= rel * np.abs(ref) + 4e-6 * g + 1e-30)
+
+
+@pytest.mark.parametrize("unroll", [None, 4, 6, 8])
+def test_k2_peeled_long_rows_every_unroll(unroll):
+    """Long rows off a 16-byte boundary (V = 151937 bf16, odd row stride) run
+    the peeled 512-thread kernel; each number of vectors in flight gives the
+    oracle's results on every token."""
+    T, V = 24, 151937
+    g = torch.Generator(device="cuda").manual_seed(11)
+    z = (torch.randn((T, V), generator=g, device="cuda") * 2.5).to(torch.bfloat16)
+    zo = (z.float() + 0.3 * torch.randn((T, V), generator=g, device="cuda")).to(torch.bfloat16)
+    ids = torch.randint(0, V, (T,), generator=g, device="cuda", dtype=torch.int32)
+    ids[0], ids[-1] = 0, V - 1
+    rows = np.arange(T)
+    lo64, _ = logprob_rows(zo, ids, rows)
+    lt64, lse = logprob_rows(z, ids, rows)
+    from paper_2605_12070_gb300.workloads import LossBatch
+    b = LossBatch(name="peeled", z_theta=z, z_old=zo, ids=ids,
+                  logp_mu=torch.from_numpy(fp32(lo64 + np.random.default_rng(11).normal(0, 0.3, T))).cuda(),
+                  adv=torch.randn(T, generator=g, device="cuda"),
+                  mask=(torch.rand(T, generator=g, device="cuda") < 0.8).to(torch.uint8),
+                  rd_lo=0.7, rd_hi=1.4, eps_low=0.2, eps_high=0.28)
+    assert z.stride(0) % 2 == 1
+    o = oracle_loss(b, lt64, fp32(lo64), loss_params(b))
+    shape = {} if unroll is None else dict(k2_threads=512, k2_unroll=unroll)
+    with occ.options(**shape):
+        out = occ.occ_decoupled_loss_fwd_bwd(z, ids, torch.from_numpy(fp32(lo64)).cuda(), b.logp_mu,
+                                             b.adv, b.mask, **b.thresholds())
+        assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    torch.cuda.synchronize()
+    s = occ.decode_loss_stats(out["stats"])
+    near = np.minimum(o["dist_rd"], o["dist_rs"]) <= 1e-6
+    assert not ((out["flags"].cpu().numpy() != o["flags"]) & ~near).any()
+    assert abs(s.loss - o["loss"]) <= 1e-4 * abs(o["loss"]) + 1e-12
+    v = o["valid"]
+    assert np.abs(out["logp"].cpu().numpy()[v] - lt64[v]).max() <= 1e-5
+    ref = dlogits_rows(b, rows, lse, o["g"])
+    got = out["dlogits"].float().cpu().numpy()
+    g_ = np.abs(o["g"])[:, None]
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 4e-6 * g_ + 1e-30)
