@@ -136,7 +136,8 @@ typedef struct {
  *   ids      [T] int32 sampled token ids
  *   logp_out [T] float32 (written); NaN where ids[t] is outside [0, V)
  *   lse_out  [T] float32 or NULL
- * Accumulation is float32 per element with a float64 row epilogue.
+ * Accumulation is float32 per element; the row epilogue works in float-float
+ * (unevaluated sums of two floats, about 48 significant bits).
  */
 occ_status occ_token_logprob(const void* logits, occ_dtype dt, int64_t T, int64_t V, int64_t ld,
                              const int32_t* ids, float* logp_out, float* lse_out, void* stream);
@@ -158,7 +159,8 @@ size_t occ_loss_workspace_bytes(int64_t T, int64_t V);
  *   loss     = sum_t loss_t / N,  N = sum_t m_t (or params->denom)
  *   dlogits[t, v] = g_t (1[v = ids[t]] - softmax(logits[t])_v),
  *   g_t      = -grad_scale m_t M_d MIS_ppo w_d r_s A_t / N
- * Threshold decisions are taken in log-ratio space in float64.
+ * Threshold decisions are taken in log-ratio space in float-float arithmetic
+ * (about 48 significant bits; the proxies of Table 1 are formed in float64).
  *
  *   logits     [T, ld] bf16 or f32 (dt); read once
  *   ids        [T] int32;  logp_old, logp_mu, adv: [T] float32 (logp_old may be NULL when
@@ -191,7 +193,7 @@ occ_status occ_decoupled_loss_fwd_bwd(const void* logits, occ_dtype dt, int64_t 
  * Each token's old row (pi_old, or the proxy pi_prox of Eq. 5 / pi_async of
  * Table 1) and current row are streamed by the same CTA, so log pi_old(y_t)
  * never leaves the kernel and enters the r_d / r_s decisions (Eqs. 1-4) in
- * float64; the old row of a dropped token (mask 0 or bad id) is not read.
+ * float-float; the old row of a dropped token (mask 0 or bad id) is not read.
  * Results equal the two-call sequence up to that float32 rounding of log pi_old.
  * Optionally, in the same pass and with no extra memory traffic, per-token
  * diagnostics of the proximal reference's lag (Sec. 5.2, App. E):

@@ -282,16 +282,63 @@ __device__ __forceinline__ void block_lse(const LseAcc& a, RedScratch& r, float&
   C = Cb;
 }
 
-// Row epilogue in float64: lse from the merged (C, S).  The terms were
-// 2^(z L - C) with L = float(log2 e); dividing the base-2 result by that same
-// L keeps the error at float(log2 e)'s relative error times the row entropy.
-__device__ __forceinline__ double lse_from(float C, float2 S) {
-  if (!(S.x > 0.f)) return (S.x == 0.f) ? -INFINITY : (double)NAN;
+// ------------------------------------------------------ float-float scalars
+
+// Per-row scalars (log-sum-exp, log-probabilities, log-ratios) are unevaluated
+// sums hi + lo of two floats with |lo| <= ulp(hi) / 2: about 48 significant
+// bits from float32 operations (Dekker 1971; Knuth, TAOCP vol. 2, 4.2.2, the
+// same TwoSum as pair_add).  The row epilogue runs in one thread while the rest
+// of the CTA waits, and a float64 instruction issues at a small fraction of the
+// float32 rate on GB300: the float64 epilogue of the fused kernel took ~4700
+// cycles per row.  Non-finite values carry lo = 0.
+struct ff {
+  float hi, lo;
+};
+
+// a + b = s + e exactly (TwoSum).
+__device__ __forceinline__ ff ff_two_sum(float a, float b) {
+  const float s = a + b;
+  const float bp = s - a;
+  const float e = (a - (s - bp)) + (b - bp);
+  return {s, isfinite(s) ? e : 0.f};
+}
+__device__ __forceinline__ ff ff_neg(ff a) { return {-a.hi, -a.lo}; }
+__device__ __forceinline__ ff ff_add(ff a, float b) {
+  const ff s = ff_two_sum(a.hi, b);
+  return ff_two_sum(s.hi, s.lo + a.lo);
+}
+__device__ __forceinline__ ff ff_sub(ff a, ff b) {
+  const ff s = ff_two_sum(a.hi, -b.hi);
+  return ff_two_sum(s.hi, s.lo + (a.lo - b.lo));
+}
+// a b with the exact error of hi * hi from one FMA.
+__device__ __forceinline__ ff ff_mul(ff a, ff b) {
+  const float p = a.hi * b.hi;
+  const float e = fmaf(a.hi, b.hi, -p);
+  return ff_two_sum(p, fmaf(a.hi, b.lo, fmaf(a.lo, b.hi, e)));
+}
+// a <= b for normalised pairs; false when either is NaN.
+__device__ __forceinline__ bool ff_le(ff a, ff b) {
+  return a.hi < b.hi || (a.hi == b.hi && a.lo <= b.lo);
+}
+__device__ __forceinline__ float ff_round(ff a) { return a.hi + a.lo; }
+
+// 1 / float(log2 e) as a float-float constant.
+constexpr float kInvLog2eHi = (float)kInvLog2eF;
+constexpr float kInvLog2eLo = (float)(kInvLog2eF - (double)kInvLog2eHi);
+
+// Row epilogue: log2 of the row's sum of exponentials from the merged (C, S),
+// in the base-2 units of the terms 2^(z L - C), L = float(log2 e).
+__device__ __forceinline__ ff lse2_from(float C, float2 S) {
+  if (!(S.x > 0.f)) return {(S.x == 0.f) ? -INFINITY : __int_as_float(0x7fc00000), 0.f};
   int e;
   const float f = frexpf(S.x, &e);  // S.x = f 2^e, f in [0.5, 1)
-  const double l2 = (double)C + (double)e + (double)log2f(f) +
-                    (double)(S.y / S.x) * 1.4426950408889634;
-  return l2 * kInvLog2eF;
+  ff l = ff_two_sum(C, (float)e);
+  l = ff_add(l, log2f(f));
+  return ff_add(l, __fdividef(S.y, S.x) * 1.4426950408889634f);  // a correction ~1e-8 of S.x
 }
+// The natural-log lse: the base-2 value divided by that same L keeps the error
+// at float(log2 e)'s relative error times the row entropy.
+__device__ __forceinline__ ff lse_nat(ff l2) { return ff_mul(l2, ff{kInvLog2eHi, kInvLog2eLo}); }
 
 }  // namespace occ

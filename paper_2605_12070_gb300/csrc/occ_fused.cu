@@ -33,6 +33,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ FusedRed red;
   __shared__ float bc_g, bc_cb;
+  __shared__ FusedTok tk_sm;  // thread 0's token scalars, kept over the broadcast
   const K2Args& a = f.a;
   const uint64_t keep = l2_policy_evict_last();
   const uint64_t last = l2_policy_evict_first();
@@ -114,13 +115,16 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
     float C[2], SV[2];
     float2 S[2];
     block_lse_v2<NT>(acc, red, C, S, SV);
-    if (tid == 0) {
+    if (tid < 32) {
       float g, cb;
-      fused_token_epilogue(f, row, C, S, SV, zy, zyo, lpm, A, N, g, cb);
-      bc_g = g;
-      bc_cb = cb;
+      fused_token_epilogue(f, C, S, zy, zyo, lpm, A, N, tid, g, cb, tk_sm);
+      if (tid == 0) {
+        bc_g = g;
+        bc_cb = cb;
+      }
     }
     __syncthreads();
+    if (tid == 0) fused_token_outputs(f, row, tk_sm, S, SV);
     if (drow) {
       const float g = bc_g, cb = bc_cb;
       if (g == 0.f) {
@@ -170,6 +174,7 @@ template <typename Tin, typename Tout, int NT, bool DIAG>
 __global__ void __launch_bounds__(NT) k2_fused_stream(const FusedArgs f) {
   __shared__ FusedRed red;
   __shared__ float bc_g, bc_cb;
+  __shared__ FusedTok tk_sm;  // thread 0's token scalars, kept over the broadcast
   const K2Args& a = f.a;
   const int tid = threadIdx.x;
   const int64_t V = a.V;
@@ -211,13 +216,16 @@ __global__ void __launch_bounds__(NT) k2_fused_stream(const FusedArgs f) {
     float C[2], SV[2];
     float2 S[2];
     block_lse_v2<NT>(acc, red, C, S, SV);
-    if (tid == 0) {
+    if (tid < 32) {
       float g, cb;
-      fused_token_epilogue(f, row, C, S, SV, zy, zyo, lpm, A, N, g, cb);
-      bc_g = g;
-      bc_cb = cb;
+      fused_token_epilogue(f, C, S, zy, zyo, lpm, A, N, tid, g, cb, tk_sm);
+      if (tid == 0) {
+        bc_g = g;
+        bc_cb = cb;
+      }
     }
     __syncthreads();
+    if (tid == 0) fused_token_outputs(f, row, tk_sm, S, SV);
     if (drow) {
       const float g = bc_g, cb = bc_cb;
       const float sgn = g > 0.f ? -1.f : 1.f;

@@ -24,38 +24,50 @@ __device__ __forceinline__ void fused_dropped_outputs(const FusedArgs& f, int64_
   if (f.kl_out) f.kl_out[row] = 0.f;
 }
 
-// Thread 0: token scalars from the two merged rows.  Writes the per-token
-// outputs and returns (g, cb) for the backward pass.
-__device__ __forceinline__ void fused_token_epilogue(const FusedArgs& f, int64_t row,
-                                                     const float (&C)[2], const float2 (&S)[2],
-                                                     const float (&SV)[2], float zy, float zyo,
-                                                     float lpm, float A, long long N, float& g,
-                                                     float& cb) {
-  const K2Args& a = f.a;
-  const double lse = lse_from(C[0], S[0]);
-  const double lse_old = lse_from(C[1], S[1]);
-  const double logp_old = (double)zyo - lse_old;
+// What the per-token outputs need after the backward pass's scalars are out.
+struct FusedTok {
+  ff lse, lse_old, logp_old;
   float loss_t, logp_f;
-  uint32_t fl;
-  token_math(a.kp, lse, zy, logp_old, lpm, A, N, g, loss_t, fl, logp_f);
-  cb = 0.f;
-  if (g != 0.f) {
-    int e;
-    const float fm = frexpf(fabsf(g), &e);
-    cb = (float)(lse * (double)kLog2e - (double)e - (double)log2f(fm));
+  uint32_t flags;
+};
+
+// Warp 0, after the CTA merge (C, S valid in every lane): lanes 0 and 1 form
+// the current and the old row's log-sum-exp side by side, then lane 0 the
+// token scalars and the backward pass's (g, cb).  Only what the backward pass
+// waits for is done here; the outputs follow in fused_token_outputs.
+__device__ __forceinline__ void fused_token_epilogue(const FusedArgs& f, const float (&C)[2],
+                                                     const float2 (&S)[2], float zy, float zyo,
+                                                     float lpm, float A, long long N, int lane,
+                                                     float& g, float& cb, FusedTok& tk) {
+  const bool old_row = lane == 1;
+  const ff l2 = lse2_from(old_row ? C[1] : C[0], old_row ? S[1] : S[0]);
+  const ff l = lse_nat(l2);
+  const ff lo = {__shfl_sync(0xffffffffu, l.hi, 1), __shfl_sync(0xffffffffu, l.lo, 1)};
+  if (lane != 0) return;
+  tk.lse = l;
+  tk.lse_old = lo;
+  tk.logp_old = ff_add(ff_neg(lo), zyo);
+  token_math(f.a.kp, l, zy, tk.logp_old, lpm, A, N, g, tk.loss_t, tk.flags, tk.logp_f);
+  cb = backward_offset(l2, g);
+}
+
+// Thread 0, while the CTA writes dlogits: the per-token outputs.
+__device__ __forceinline__ void fused_token_outputs(const FusedArgs& f, int64_t row,
+                                                    const FusedTok& tk, const float2 (&S)[2],
+                                                    const float (&SV)[2]) {
+  const K2Args& a = f.a;
+  a.ws_loss[row] = tk.loss_t;
+  a.ws_flags[row] = (uint8_t)tk.flags;
+  if (a.logp_out) a.logp_out[row] = tk.logp_f;
+  if (a.flags_out) a.flags_out[row] = (uint8_t)tk.flags;
+  if (f.logp_old_out) f.logp_old_out[row] = ff_round(tk.logp_old);
+  if (f.entropy_out) {  // H = lse - E_p[z]
+    const float ez = SV[0] / (S[0].x + S[0].y);
+    f.entropy_out[row] = ff_round(ff_add(tk.lse, -ez));
   }
-  a.ws_loss[row] = loss_t;
-  a.ws_flags[row] = (uint8_t)fl;
-  if (a.logp_out) a.logp_out[row] = logp_f;
-  if (a.flags_out) a.flags_out[row] = (uint8_t)fl;
-  if (f.logp_old_out) f.logp_old_out[row] = (float)logp_old;
-  if (f.entropy_out) {
-    const double ez = (double)SV[0] / ((double)S[0].x + (double)S[0].y);
-    f.entropy_out[row] = (float)(lse - ez);
-  }
-  if (f.kl_out) {
-    const double ed = (double)SV[1] / ((double)S[1].x + (double)S[1].y);
-    f.kl_out[row] = (float)(ed - lse_old + lse);
+  if (f.kl_out) {  // KL = E_{p_old}[z_old - z] - lse_old + lse
+    const float ed = SV[1] / (S[1].x + S[1].y);
+    f.kl_out[row] = ff_round(ff_add(ff_sub(tk.lse, tk.lse_old), ed));
   }
 }
 

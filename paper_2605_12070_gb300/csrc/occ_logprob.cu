@@ -64,9 +64,9 @@ __global__ void __launch_bounds__(NT, 1024 / NT)
     float2 S;
     block_lse<NT>(acc, red, C, S);
     if (threadIdx.x == 0) {
-      const double l = lse_from(C, S);
-      logp[row] = (id >= 0 && id < V) ? (float)((double)zy - l) : __int_as_float(0x7fc00000);
-      if (lse_out) lse_out[row] = (float)l;
+      const ff l = lse_nat(lse2_from(C, S));
+      logp[row] = (id >= 0 && id < V) ? ff_round(ff_add(ff_neg(l), zy)) : __int_as_float(0x7fc00000);
+      if (lse_out) lse_out[row] = ff_round(l);
     }
     __syncthreads();
   }
@@ -117,9 +117,9 @@ __global__ void __launch_bounds__(NT, 1024 / NT)
       const int id = ids[row];
       const bool ok = id >= 0 && id < V;
       const float zy = ok ? Elem<Tin>::load(z0 + id) : 0.f;
-      const double l = lse_from(C, S);
-      logp[row] = ok ? (float)((double)zy - l) : __int_as_float(0x7fc00000);
-      if (lse_out) lse_out[row] = (float)l;
+      const ff l = lse_nat(lse2_from(C, S));
+      logp[row] = ok ? ff_round(ff_add(ff_neg(l), zy)) : __int_as_float(0x7fc00000);
+      if (lse_out) lse_out[row] = ff_round(l);
     }
   }
 }
@@ -154,9 +154,9 @@ __global__ void __launch_bounds__(NT)
     float2 S;
     block_lse<NT>(acc, red, C, S);
     if (threadIdx.x == 0) {
-      const double l = lse_from(C, S);
-      logp[row] = (id >= 0 && id < V) ? (float)((double)zy - l) : __int_as_float(0x7fc00000);
-      if (lse_out) lse_out[row] = (float)l;
+      const ff l = lse_nat(lse2_from(C, S));
+      logp[row] = (id >= 0 && id < V) ? ff_round(ff_add(ff_neg(l), zy)) : __int_as_float(0x7fc00000);
+      if (lse_out) lse_out[row] = ff_round(l);
     }
     __syncthreads();
   }

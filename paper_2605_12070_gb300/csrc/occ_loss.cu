@@ -118,18 +118,12 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
     float2 Sr;
     block_lse<NT>(acc, red, Cr, Sr);
     if (tid == 0) {
-      const double lse = lse_from(Cr, Sr);
+      const ff l2 = lse2_from(Cr, Sr);
       float g, loss_t, logp_f;
       uint32_t fl;
-      token_math(a.kp, lse, zy, lpo, lpm, A, N, g, loss_t, fl, logp_f);
-      float cb = 0.f;
-      if (g != 0.f) {
-        int e;
-        const float fm = frexpf(fabsf(g), &e);
-        cb = (float)(lse * (double)kLog2e - (double)e - (double)log2f(fm));
-      }
+      token_math(a.kp, lse_nat(l2), zy, ff{lpo, 0.f}, lpm, A, N, g, loss_t, fl, logp_f);
       bc_g = g;
-      bc_cb = cb;
+      bc_cb = backward_offset(l2, g);
       a.ws_loss[row] = loss_t;
       a.ws_flags[row] = (uint8_t)fl;
       if (a.logp_out) a.logp_out[row] = logp_f;
@@ -223,13 +217,13 @@ __global__ void __launch_bounds__(NT) k2_loss_stream(const K2Args a) {
   float2 Sr;
   block_lse<NT>(acc, red, Cr, Sr);
   if (tid == 0) {
-    const double lse = lse_from(Cr, Sr);
+    const ff l2 = lse2_from(Cr, Sr);
     const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
     float g, loss_t, logp_f;
     uint32_t fl;
-    token_math(a.kp, lse, zy, lpo, lpm, A, N, g, loss_t, fl, logp_f);
+    token_math(a.kp, lse_nat(l2), zy, ff{lpo, 0.f}, lpm, A, N, g, loss_t, fl, logp_f);
     bc_g = g;
-    bc_cb = (float)(lse * (double)kLog2e);
+    bc_cb = ff_round(l2);
     a.ws_loss[row] = loss_t;
     a.ws_flags[row] = (uint8_t)fl;
     if (a.logp_out) a.logp_out[row] = logp_f;

@@ -5,6 +5,8 @@
 
 #include <math.h>
 
+#include <cmath>
+
 #include "occ_common.cuh"
 
 namespace occ {
@@ -15,8 +17,8 @@ constexpr int kFinThreads = 1024;
 constexpr uint8_t kWsBadId = 0x80;           // workspace flag: dropped for a bad id
 
 struct LossKParams {
-  double log_rd_lo, log_rd_hi;    // log of the r_d band (may be -inf / +inf)
-  double log_clip_lo, log_clip_hi;  // log(1 - eps_low), log(1 + eps_high)
+  ff log_rd_lo, log_rd_hi;        // log of the r_d band (may be -inf / +inf), float-float
+  ff log_clip_lo, log_clip_hi;    // log(1 - eps_low), log(1 + eps_high), float-float
   float clip_lo, clip_hi;         // 1 - eps_low, 1 + eps_high
   float grad_scale;
   int rd_weight;
@@ -58,27 +60,42 @@ struct K2Args {
   LossKParams kp;
 };
 
-// Per-token scalar part (R2..R8): threshold decisions in float64 log space.
-__device__ __forceinline__ void token_math(const LossKParams& kp, double lse, float zy, double lpo,
+// Per-token scalar part (R2..R8): threshold decisions in float-float log space
+// (the proxies of Table 1 are formed in float64: log1p / expm1).
+__device__ __forceinline__ void token_math(const LossKParams& kp, ff lse, float zy, ff lpo,
                                            float lpm, float A, long long N, float& g,
                                            float& loss_t, uint32_t& flags, float& logp_f) {
-  const double logp = (double)zy - lse;
-  if (kp.proxy != OCC_PROXY_NONE) lpo = proxy_logprob(kp.proxy, kp.alpha, (double)lpm, logp);
-  const double log_rd = (double)lpo - (double)lpm;
-  const bool in_band = (log_rd >= kp.log_rd_lo) && (log_rd <= kp.log_rd_hi);
-  const double log_rs = logp - (double)lpo;
-  const bool mis = (A >= 0.f) ? (log_rs <= kp.log_clip_hi) : (log_rs >= kp.log_clip_lo);
-  const float r_s = expf((float)log_rs);
-  const float r_d = expf((float)log_rd);
+  const ff logp = ff_add(ff_neg(lse), zy);
+  if (kp.proxy != OCC_PROXY_NONE) {
+    const double d = proxy_logprob(kp.proxy, kp.alpha, (double)lpm, (double)logp.hi + (double)logp.lo);
+    const float h = (float)d;
+    lpo = ff{h, isfinite(h) ? (float)(d - (double)h) : 0.f};
+  }
+  const ff log_rd = ff_add(lpo, -lpm);
+  const bool in_band = ff_le(kp.log_rd_lo, log_rd) && ff_le(log_rd, kp.log_rd_hi);
+  const ff log_rs = ff_sub(logp, lpo);
+  const bool mis = (A >= 0.f) ? ff_le(log_rs, kp.log_clip_hi) : ff_le(kp.log_clip_lo, log_rs);
+  const float r_s = expf(ff_round(log_rs));
+  const float r_d = expf(ff_round(log_rd));
   const float w = kp.rd_weight ? r_d : 1.f;
   const float rc = fminf(fmaxf(r_s, kp.clip_lo), kp.clip_hi);
   const float s = fminf(r_s * A, rc * A);
   const bool active = in_band && mis;
   loss_t = in_band ? -w * s : 0.f;
-  g = (active && N > 0) ? (-kp.grad_scale * w * r_s * A) / (float)N : 0.f;
+  g = (active && N > 0) ? __fdividef(-kp.grad_scale * w * r_s * A, (float)N) : 0.f;
   flags = (in_band ? OCC_FLAG_IN_BAND : 0) | (mis ? 0 : OCC_FLAG_CLIPPED) |
           (active ? OCC_FLAG_ACTIVE : 0) | OCC_FLAG_VALID;
-  logp_f = (float)logp;
+  logp_f = ff_round(logp);
+}
+
+// Exponent offset of the backward pass, g folded in: dlogits_v = -sign(g)
+// 2^(z_v L - cb) (+ g at the sampled token) with cb = lse L - log2|g|, from the
+// base-2 lse l2; 0 when g = 0.
+__device__ __forceinline__ float backward_offset(ff l2, float g) {
+  if (g == 0.f) return 0.f;
+  int e;
+  const float fm = frexpf(fabsf(g), &e);  // |g| = fm 2^e
+  return ff_round(ff_add(ff_add(l2, -(float)e), -log2f(fm)));
 }
 
 // Writes VEC gradient values starting at a 16-byte aligned output address.
@@ -388,6 +405,12 @@ __device__ __forceinline__ void block_lse_v2(const LseAccV (&acc)[2], FusedRed& 
 }
 
 
+// Host: a double threshold as a normalised float-float pair.
+inline ff ff_of(double x) {
+  const float h = (float)x;
+  return ff{h, std::isfinite(h) ? (float)(x - (double)h) : 0.f};
+}
+
 // Host: validates the arguments every loss entry point shares (all but the
 // source of log pi_old), fills the kernel arguments and reports whether the
 // rows qualify for the 16-byte vector kernels.
@@ -462,10 +485,10 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   a.flags_out = flags_out;
   a.dlogits = dlogits;
   a.ld_grad = ld_grad;
-  a.kp.log_rd_lo = p->rd_lo > 0.0 ? log(p->rd_lo) : -INFINITY;
-  a.kp.log_rd_hi = isinf(p->rd_hi) ? INFINITY : log(p->rd_hi);
-  a.kp.log_clip_lo = p->eps_low < 1.0 ? log1p(-p->eps_low) : -INFINITY;
-  a.kp.log_clip_hi = log1p(p->eps_high);
+  a.kp.log_rd_lo = ff_of(p->rd_lo > 0.0 ? log(p->rd_lo) : -INFINITY);
+  a.kp.log_rd_hi = ff_of(isinf(p->rd_hi) ? INFINITY : log(p->rd_hi));
+  a.kp.log_clip_lo = ff_of(p->eps_low < 1.0 ? log1p(-p->eps_low) : -INFINITY);
+  a.kp.log_clip_hi = ff_of(log1p(p->eps_high));
   a.kp.clip_lo = (float)(1.0 - p->eps_low);
   a.kp.clip_hi = (float)(1.0 + p->eps_high);
   a.kp.grad_scale = (float)p->grad_scale;
