@@ -52,6 +52,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--tau", type=float, default=0.5)
     ap.add_argument("--tokens", type=int, default=None, help="resize T (profiling runs only)")
+    ap.add_argument("--vocab", type=int, default=None,
+                    help="resize V (profiling runs only; an odd V puts the bf16 rows off 16-byte "
+                         "boundaries, which the peeled kernels take)")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="loss batch (default: the agentic batch the metric is quoted on; the "
                          "others are for breakdowns only)")
@@ -425,7 +428,7 @@ def main():
         dev = torch.device(f"cuda:{local}" if torch.cuda.is_available() else "cpu")
         if dev.type == "cuda":
             torch.cuda.set_device(dev)
-        batch = make_loss_batch(args.workload, T=args.tokens, seed=0, device=dev)
+        batch = make_loss_batch(args.workload, T=args.tokens, V=args.vocab, seed=0, device=dev)
         run_reference(args, batch, world)
         return
     if world > 1:
@@ -439,7 +442,7 @@ def main():
     from paper_2605_12070_gb300 import dp, occ
     from paper_2605_12070_gb300.workloads import make_ewma_buffers, make_loss_batch
 
-    batch = make_loss_batch(args.workload, T=args.tokens, seed=rank, device=dev)
+    batch = make_loss_batch(args.workload, T=args.tokens, V=args.vocab, seed=rank, device=dev)
     T, V = batch.T, batch.V
     n_valid = T if batch.mask is None else int(batch.mask.sum().item())
 
