@@ -7,7 +7,7 @@
 // exponent c only moves when a new value exceeds it by more than kRescale
 // (lazy rescaling), so the inner loop is one FFMA, one MUFU.EX2 and one FADD
 // per element.  Partials are merged with one accurate exp2f per thread and a
-// compensated (two-float) tree sum, and the row epilogue runs in float64.
+// compensated (two-float) tree sum, and the row epilogue runs in float-float.
 #pragma once
 
 #include <cuda_runtime.h>

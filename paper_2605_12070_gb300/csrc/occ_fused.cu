@@ -4,7 +4,7 @@
 // One CTA per row streams the old (or proxy) logits row and the current
 // logits row side by side in the forward pass: log pi_old(y_t) and
 // log pi_theta(y_t) come out of the same CTA (Eq. 1 factors), log pi_old stays
-// in float64 into the ratio decisions (Eqs. 2-4), and the old row of a dropped
+// in float-float into the ratio decisions (Eqs. 2-4), and the old row of a dropped
 // token is never read.  The backward pass is the K2 one (the current row's
 // head from shared memory, the rest re-read from L2).
 //
