@@ -249,37 +249,39 @@ __device__ __forceinline__ float2 warp_pair_sum(float2 v) {
 
 // Shared scratch for block reductions (one slot per warp).
 struct RedScratch {
-  float m[32];
+  float c[32];
   float2 s[32];
-  float bc;
 };
 
-// Merges the per-thread (c, s) of a block.  Result (C, S) is valid in thread 0:
+// Merges the per-thread (c, s) of a block with one barrier: each warp scales
+// its sum to the warp's largest reference exponent, then warp 0 merges the
+// warps' pairs (compensated).  Result (C, S) is valid in every lane of warp 0:
 // sum over the block of 2^(z L - C) = S.x + S.y.  Deterministic order.
 template <int NT>
 __device__ __forceinline__ void block_lse(const LseAcc& a, RedScratch& r, float& C, float2& S) {
   constexpr int NW = NT / 32;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  float m = warp_max(a.c);
-  if (lane == 0) r.m[wid] = m;
-  __syncthreads();
-  if (wid == 0) {
-    float v = lane < NW ? r.m[lane] : -INFINITY;
-    v = warp_max(v);
-    if (lane == 0) r.bc = v;
+  const float wm = warp_max(a.c);
+  const float f = a.c == -INFINITY ? 0.f : exp2f(a.c - wm);
+  const float2 v = warp_pair_sum(make_float2(a.s * f, 0.f));
+  if (lane == 0) {
+    r.c[wid] = wm;
+    r.s[wid] = v;
   }
   __syncthreads();
-  const float Cb = r.bc;
-  float2 v = make_float2((a.c == -INFINITY) ? 0.f : a.s * exp2f(a.c - Cb), 0.f);
-  v = warp_pair_sum(v);
-  if (lane == 0) r.s[wid] = v;
-  __syncthreads();
   if (wid == 0) {
-    float2 w = lane < NW ? r.s[lane] : make_float2(0.f, 0.f);
-    w = warp_pair_sum(w);
-    if (lane == 0) S = w;
+    const float cw = lane < NW ? r.c[lane] : -INFINITY;
+    const float cm = warp_max(cw);
+    float2 w = make_float2(0.f, 0.f);
+    if (lane < NW && cw != -INFINITY) {
+      const float g = exp2f(cw - cm);
+      const float2 p = r.s[lane];
+      const float hi = p.x * g;
+      w = make_float2(hi, fmaf(p.x, g, -hi) + p.y * g);
+    }
+    S = warp_pair_sum(w);
+    C = cm;
   }
-  C = Cb;
 }
 
 // ------------------------------------------------------ float-float scalars
