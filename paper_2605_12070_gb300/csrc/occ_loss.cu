@@ -245,9 +245,10 @@ __global__ void __launch_bounds__(NT) k2_loss_stream(const K2Args a) {
 
 using K2Kern = void (*)(const K2Args);
 
-// Vectors in flight per thread of the 512-thread tier: 8 for aligned rows, 6
-// for peeled ones (V = 151937, GB300: 6.41 ms against 6.77 with 8, which
-// spills, and 6.55 with 4); `unroll` > 0 overrides.
+// Vectors in flight per thread of the 512-thread tier: 8 for aligned rows
+// (V = 151936, GB300: 5.92 ms against 6.08 with 6), 6 for peeled ones
+// (V = 151937: 6.20 ms against 6.46 with 8 and 6.50 with 4); `unroll` > 0
+// overrides.
 template <typename Tin, typename Tout, bool PEEL>
 static K2Kern l2_kernel(int nt, int unroll) {
   const int u = unroll > 0 ? unroll : (PEEL ? 6 : 8);
