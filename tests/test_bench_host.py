@@ -67,6 +67,34 @@ def test_traffic_is_used_only_for_the_captured_batch(tmp_path):
     assert bench.traffic_bytes(tr, "k1_token_logprob", T=20, n_valid=10, n_params=0) is None
 
 
+def test_partial_capture_keeps_unchanged_kernels_and_drops_stale_ones(tmp_path):
+    # a capture of one kernel rewrites its entry and keeps the others while their
+    # sources hash as recorded; an entry whose hash no longer matches is dropped
+    import json
+    path = str(tmp_path / "traffic.json")
+    both = tmp_path / "both.csv"
+    _fake_csv(both, [("void k2_loss_l2<bf16_t, bf16_t, 512, 8, 0>(K2Args)", m, "byte", "1000")
+                     for m in ("dram__bytes_read.sum", "dram__bytes_write.sum")]
+              + [("void k3_ewma_vec<256, 4>(x)", m, "byte", "1000")
+                 for m in ("dram__bytes_read.sum", "dram__bytes_write.sum")])
+    bench.write_traffic(str(both), "agentic_bf16_v151936", 151936, 10, 5, 100, "cmd", path=path)
+    one = tmp_path / "one.csv"
+    _fake_csv(one, [("void k3_ewma_vec<256, 4>(x)", m, "byte", "3000")
+                    for m in ("dram__bytes_read.sum", "dram__bytes_write.sum")])
+    out = bench.write_traffic(str(one), "agentic_bf16_v151936", 151936, 10, 5, 100, "cmd", path=path)
+    assert set(out["kernels"]) == {"k2_decoupled_loss_fwd_bwd", "k3_ewma_update"}
+    assert out["kernels"]["k3_ewma_update"]["read_per_param"] == 30.0
+    assert out["kernels"]["k2_decoupled_loss_fwd_bwd"]["read_per_valid_token"] == 200.0
+    d = json.load(open(path))
+    d["kernels"]["k2_decoupled_loss_fwd_bwd"]["source_hash"] = "stale"
+    json.dump(d, open(path, "w"))
+    out = bench.write_traffic(str(one), "agentic_bf16_v151936", 151936, 10, 5, 100, "cmd", path=path)
+    assert set(out["kernels"]) == {"k3_ewma_update"}
+    # a capture of another batch starts a new table
+    out = bench.write_traffic(str(one), "grpo_bf16_v32000", 32000, 10, 5, 100, "cmd", path=path)
+    assert set(out["kernels"]) == {"k3_ewma_update"} and out["workload"] == "grpo_bf16_v32000"
+
+
 def test_shared_workload_config_keys():
     class A:
         workload, ewma_n, tau = "agentic_bf16_v151936", 100, 0.5
