@@ -369,7 +369,8 @@ typedef enum {
   OCC_OPT_K2_UNROLL = 4,       /* vectors in flight per thread of its 512-thread kernel: 4, 6, 8 */
   OCC_OPT_FUSED_THREADS = 5,   /* threads per occ_decoupled_loss_fused CTA: 128, 256, 512 */
   OCC_OPT_FUSED_HEAD_BYTES = 6, /* its shared-memory head, bytes                       */
-  OCC_OPT_COUNT_ = 7
+  OCC_OPT_FUSED_TMEM = 7,      /* 0: no tensor-memory row cache for long rows; 1: allowed */
+  OCC_OPT_COUNT_ = 8
 } occ_option;
 occ_status occ_set_option(occ_option opt, int64_t value);
 int64_t occ_get_option(occ_option opt);

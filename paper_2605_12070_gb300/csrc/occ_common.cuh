@@ -169,6 +169,53 @@ __device__ __forceinline__ void acc_add_fast(LseAcc& a, const float (&x)[N]) {
     acc_add(a, x);
 }
 
+// ------------------------------------------------------- tensor memory (TMEM)
+
+// Tensor memory is the 256 KB per SM (128 lanes x 512 columns of 32 bits) that
+// tcgen05 matrix instructions accumulate into.  No step of this path is a
+// contraction, so the loss kernels use it as plain on-chip storage for part of
+// a logits row.  A warp reaches only its quarter of the lanes (warp % 4); each
+// thread owns one lane, and a 32x32b.x4 access moves 16 bytes per thread to or
+// from 4 consecutive columns of that lane.  Allocation is per CTA, by one warp.
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(dst_smem)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+// Orders tcgen05 work around a CTA barrier (the allocation's address, the
+// last accesses before the deallocation).
+__device__ __forceinline__ void tmem_fence_before_sync() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_fence_after_sync() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint4& v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr),
+               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ uint4 tmem_ld16(uint32_t taddr) {
+  uint4 v;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(taddr)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
 // ------------------------------------------------------------ row streaming
 
 // How a thread walks the vectors i = t, t + NT, t + 2 NT, ... < n of a row,

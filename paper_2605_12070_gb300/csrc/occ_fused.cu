@@ -8,6 +8,13 @@
 // token is never read.  The backward pass is the K2 one (the current row's
 // head from shared memory, the rest re-read from L2).
 //
+// Long rows (the 512-thread tier) keep more of the current row on chip: a
+// shared-memory head and, after it, 128 KB in tensor memory, which no step of
+// this path needs for matrix work.  Only the rest of the row is re-read from L2,
+// and the re-reads that the gradient writes would push out of L2 are gone.  That
+// kernel is persistent (two CTAs per SM, rows fetched from a counter), so each
+// CTA allocates its tensor memory once.
+//
 // Diagnostics (optional, no extra HBM bytes): the entropy of pi_theta,
 // H = lse - E_p[z], and KL(pi_old || pi_theta) = E_{p_old}[z_old - z] -
 // lse_old + lse, which track the reference-policy lag that the revised
@@ -18,6 +25,16 @@
 
 namespace occ {
 
+// The tensor-memory tier (TM): rows walk in blocks of NT = 512 vectors; blocks
+// [0, kTmHeadBlocks) go to the shared-memory head (72 KB), blocks
+// [kTmHeadBlocks, kTmHeadBlocks + kTmBlocks) to tensor memory (128 KB: 256
+// columns of the 128 lanes, two CTAs per SM take the 512 columns), the rest is
+// re-read from L2.  The launcher takes this tier only for rows whose tensor-
+// memory blocks lie in full rounds of the walk.
+constexpr int kTmHeadBlocks = 9;
+constexpr int kTmBlocks = 16;
+constexpr uint32_t kTmCols = 256;
+
 // One 16-byte vector of the current row and the old row.
 struct RowPair {
   uint4 t, o;
@@ -27,20 +44,43 @@ struct RowPair {
 // PEEL: rows that start off a 16-byte boundary take their first `lead`
 // elements (up to the boundary) as scalars; the old-logits and gradient rows
 // have the same byte offset (checked on the host).
-template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL>
+template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ FusedRed red;
   __shared__ float bc_g, bc_cb;
   __shared__ FusedTok tk_sm;  // thread 0's token scalars, kept over the broadcast
+  __shared__ uint32_t tmem_sm;  // TM: the CTA's tensor-memory address
+  __shared__ long long row_sm;  // TM: the row fetched for the CTA
   const K2Args& a = f.a;
   const uint64_t keep = l2_policy_evict_last();
   const uint64_t last = l2_policy_evict_first();
   const int tid = threadIdx.x;
   const int64_t V = a.V;
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
-  for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
+  if constexpr (TM) {
+    if (tid < 32) {
+      __syncwarp();
+      tmem_alloc(&tmem_sm, kTmCols);
+    }
+    tmem_fence_before_sync();
+    __syncthreads();
+    tmem_fence_after_sync();
+  }
+  // TM: this warp's tensor memory, its quarter of the lanes and 64 of the columns
+  auto tmem_warp = [&]() {
+    return tmem_sm + ((uint32_t)(32 * ((tid >> 5) & 3)) << 16) + (uint32_t)((tid >> 5) >> 2) * 64u;
+  };
+  for (int64_t row_i = a.row0 + blockIdx.x;; row_i += gridDim.x) {
+    int64_t row = row_i;
+    if constexpr (TM) {  // rows from a counter that K0 cleared: no tail of unequal CTAs
+      __syncthreads();
+      if (tid == 0) row_sm = (long long)atomicAdd(a.ws_rows, 1u) + a.row0;
+      __syncthreads();
+      row = row_sm;
+    }
+    if (row >= a.T) break;
     const int id = a.ids[row];
     const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
     const bool id_ok = id >= 0 && (int64_t)id < V;
@@ -102,7 +142,20 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
     walk_row<kW, U, NT>(
         tid, (int)nvec,
         [&](int j) { return RowPair{ld_hint_v4(zv + j, keep), ld_hint_v4(zov + j, last)}; },
-        [&](int j, const RowPair& r) { consume(j, r.t, r.o); });
+        [&](int j, const RowPair& r) {
+          if constexpr (TM) {  // block k of the tensor-memory part: the same for the whole CTA
+            const int k = j / NT - kTmHeadBlocks;
+            if (k >= 0 && k < kTmBlocks) {
+              __syncwarp();
+              tmem_st16(tmem_warp() + 4u * (uint32_t)k, r.t);
+            }
+          }
+          consume(j, r.t, r.o);
+        });
+    if constexpr (TM) {
+      __syncwarp();
+      tmem_wait_st();
+    }
     float xt = 0.f, xp = 0.f;
     if ((int64_t)tid < ntail) {
       xt = Elem<Tin>::load(z + tail0 + tid);
@@ -145,11 +198,21 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
           }
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
-        const int64_t nre = nvec - head;
-        const uint4* zr = zv + head;
+        const int64_t rb = TM ? (int64_t)(kTmHeadBlocks + kTmBlocks) * NT : head;  // first re-read
+        const int64_t nre = nvec - rb;
+        const uint4* zr = zv + rb;
         walk_row<kW, 8, NT>(  // 8 vectors in flight, whatever the forward pass's U
             tid, (int)nre, [&](int j) { return ld_hint_v4(zr + j, last); },
-            [&](int j, const uint4& r) { emit(head + j, r); });
+            [&](int j, const uint4& r) { emit(rb + j, r); });
+        if constexpr (TM) {
+          __syncwarp();
+          const uint32_t tw = tmem_warp();
+          for (int k = 0; k < kTmBlocks; ++k) {
+            const uint4 r = tmem_ld16(tw + 4u * (uint32_t)k);
+            tmem_wait_ld();
+            emit((int64_t)(kTmHeadBlocks + k) * NT + tid, r);
+          }
+        }
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
         if ((int64_t)tid < ntail) {
@@ -165,6 +228,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
       }
     }
     __syncthreads();
+  }
+  if constexpr (TM) {
+    tmem_fence_before_sync();
+    __syncthreads();
+    tmem_fence_after_sync();
+    if (tid < 32) {
+      __syncwarp();
+      tmem_dealloc(tmem_sm, kTmCols);
+    }
   }
 }
 
@@ -300,7 +372,26 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
       if (peel) kern = fused_kernel<Tin, Tout, DIAG, true>(nt);
     const size_t head_auto =
         nt_auto == kFusedThreads ? two_cta_smem_budget((const void*)kern) : 0;
-    const size_t head = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
+    size_t head = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
+    // Long aligned rows without diagnostics take the tensor-memory tier (GB300, agentic
+    // batch V = 151936: 8.06 ms against 8.31 ms, the L2 re-read misses gone) when every
+    // tensor-memory block lies in full rounds of the walk; OCC_OPT_FUSED_TMEM = 0 or a
+    // head size from OCC_OPT_FUSED_HEAD_BYTES keeps the plain kernel.
+    bool tm = false;
+    if constexpr (!DIAG) {
+      const int64_t full_blocks = (f.a.V / Elem<Tin>::kVec) /
+                                  ((int64_t)kFusedUnroll * kFusedThreads) * kFusedUnroll;
+      if (vec && nt == kFusedThreads && option(OCC_OPT_FUSED_TMEM) != 0 && head_opt < 0 &&
+          T < step && full_blocks >= kTmHeadBlocks + kTmBlocks) {
+        FusedKern kt = k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, false, false, true>;
+        const size_t tm_head = (size_t)kTmHeadBlocks * kFusedThreads * 16;
+        if (two_cta_smem_budget((const void*)kt) >= tm_head) {
+          kern = kt;
+          head = tm_head;
+          tm = true;
+        }
+      }
+    }
     f.a.stage_bytes = (int64_t)head;
     if (head > 0) {
       cudaError_t e =
@@ -309,10 +400,16 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
         return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head,
                     cudaGetErrorString(e));
     }
-    note_kernel(peel ? "k2_fused_l2/peel" : "k2_fused_l2");
-    for (int64_t r0 = 0; r0 < T; r0 += step) {
-      f.a.row0 = r0;
-      kern<<<(unsigned)std::min<int64_t>(step, T - r0), nt, head, s>>>(f);
+    note_kernel(tm ? "k2_fused_l2/tmem" : peel ? "k2_fused_l2/peel" : "k2_fused_l2");
+    if (tm) {  // persistent: two CTAs per SM (the register limit), rows from the counter
+      f.a.row0 = 0;
+      const unsigned grid = (unsigned)std::min<int64_t>(T, (int64_t)sm_count() * 2);
+      kern<<<grid, nt, head, s>>>(f);
+    } else {
+      for (int64_t r0 = 0; r0 < T; r0 += step) {
+        f.a.row0 = r0;
+        kern<<<(unsigned)std::min<int64_t>(step, T - r0), nt, head, s>>>(f);
+      }
     }
   } else {
     note_kernel("k2_fused_stream");

@@ -45,6 +45,7 @@ struct K2Args {
   int64_t T, V, ld, S, row0;
   int64_t stage_bytes;  // bytes of the shared-memory head of the row (two-pass kernels)
   int* ws_err;          // device-detected error bits, OR-ed into stats.err
+  unsigned* ws_rows;    // row counter of the persistent fused kernel (K0 clears it)
   const int32_t* ids;
   const float* lp_old;
   const float* lp_mu;
@@ -198,9 +199,13 @@ template <int NT>
 __global__ void __launch_bounds__(NT) k0_count_valid(const uint8_t* __restrict__ mask,
                                                      const int32_t* __restrict__ ids, int64_t T,
                                                      int64_t V, long long* __restrict__ ws_N,
-                                                     int* __restrict__ ws_err) {
+                                                     int* __restrict__ ws_err,
+                                                     unsigned* __restrict__ ws_rows) {
   __shared__ long long part[NT / 32];
-  if (threadIdx.x == 0) *ws_err = 0;
+  if (threadIdx.x == 0) {
+    *ws_err = 0;
+    *ws_rows = 0;
+  }
   long long c = 0;
   for (int64_t t0 = threadIdx.x; t0 < T; t0 += 8 * (int64_t)NT) {
     int idv[8];
@@ -297,13 +302,14 @@ __global__ void __launch_bounds__(NT) k2_finalize(int64_t T, const float* __rest
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct WsLayout {
-  size_t off_N, off_err, off_loss, off_flags, total;
+  size_t off_N, off_err, off_rows, off_loss, off_flags, total;
 };
 inline WsLayout ws_layout(int64_t T) {
   const size_t t = T > 0 ? (size_t)T : 0;
   WsLayout w;
   w.off_N = 0;
   w.off_err = 8;
+  w.off_rows = 12;
   w.off_loss = 256;
   w.off_flags = w.off_loss + align_up(4 * t, 256);
   w.total = w.off_flags + align_up(t, 256);
@@ -479,6 +485,7 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
   a.mask = loss_mask;
   a.ws_N = (const long long*)(ws + wl.off_N);
   a.ws_err = (int*)(ws + wl.off_err);
+  a.ws_rows = (unsigned*)(ws + wl.off_rows);
   a.ws_loss = (float*)(ws + wl.off_loss);
   a.ws_flags = (uint8_t*)(ws + wl.off_flags);
   a.logp_out = logp_out;
@@ -505,7 +512,8 @@ inline occ_status prepare_loss_args(const void* logits, occ_dtype dt, int64_t T,
 // the workspace starts undefined).
 inline occ_status launch_k0(const K2Args& a, cudaStream_t s) {
   k0_count_valid<kK0Threads><<<1, kK0Threads, 0, s>>>(a.mask, a.ids, a.T, a.V,
-                                                      const_cast<long long*>(a.ws_N), a.ws_err);
+                                                      const_cast<long long*>(a.ws_N), a.ws_err,
+                                                      a.ws_rows);
   return check_launch("k0_count_valid");
 }
 

@@ -2,10 +2,13 @@
 (row stride V, base address 16-byte aligned), as occ_last_kernel() names it:
 the vector kernel when rows start on 16-byte boundaries, the peeled vector
 kernel when they do not but a row holds at least 16 vectors, else the
-element-load kernel; for K1, rows of up to 32 KB run one warp per row."""
+element-load kernel; for K1, rows of up to 32 KB run one warp per row.  The
+fused kernel without diagnostics runs its tensor-memory tier on aligned rows of
+the 512-thread tier (over 112 KB) that hold at least 25 blocks of 512 vectors
+in whole rounds of 4 blocks."""
 
 
-def expected_kernel(kind, V, elem_size):
+def expected_kernel(kind, V, elem_size, diag=True):
     vec = 16 // elem_size
     names = {"k1": ("k1_logprob_vec", "k1_logprob_scalar"),
              "k2": ("k2_loss_l2", "k2_loss_stream"),
@@ -14,5 +17,8 @@ def expected_kernel(kind, V, elem_size):
     if kind == "k1" and (V // vec) * 16 <= 32 * 1024:  # K1 rows up to 32 KB: one warp each
         first = "k1_logprob_warp"
     if (V * elem_size) % 16 == 0:
+        nvec = V // vec
+        if kind == "fused" and not diag and nvec * 16 > 112 * 1024 and nvec // 2048 * 4 >= 25:
+            return first + "/tmem"
         return first
     return first + "/peel" if V >= 16 * vec else names[1]

@@ -146,7 +146,7 @@ def test_fused_every_token(agentic):
     out = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
                                        **b.thresholds())
     torch.cuda.synchronize()
-    assert occ.occ_last_kernel() == "k2_fused_l2"
+    assert occ.occ_last_kernel() == "k2_fused_l2/tmem"   # the tensor-memory tier
     glo = out["logp_old"].cpu().numpy().astype(np.float64)
     st, gfl = _check_every_token(b, out, o, lt64, lo64, glo)
     assert np.all(glo[~o["valid"]] == 0.0)

@@ -1,0 +1,113 @@
+"""The fused kernel's tensor-memory tier against its plain kernel, bit for bit.
+
+Long aligned rows without diagnostics keep 128 KB of the current row in tensor
+memory instead of re-reading it from L2, and the kernel runs persistent with
+rows fetched from a counter.  The arithmetic is the plain kernel's in the same
+order, so every output must equal the plain kernel's (OCC_OPT_FUSED_TMEM = 0)
+bit for bit: dlogits, the statistics, log pi_theta, log pi_old and the flags.
+The oracle comparisons of the default path (test_gpu_fused.py,
+test_gpu_full_agentic.py) run this tier on the long-row batches.
+"""
+
+import pytest
+import torch
+
+from kernel_choice import expected_kernel
+from paper_2605_12070_gb300 import occ
+from paper_2605_12070_gb300.workloads import make_loss_batch
+
+pytestmark = pytest.mark.gpu
+
+
+def _both(b, **kw):
+    outs = []
+    for tm in (1, 0):
+        with occ.options(fused_tmem=tm):
+            out = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv,
+                                               b.mask, **b.thresholds(), **kw)
+            kern = occ.occ_last_kernel()
+        torch.cuda.synchronize()
+        outs.append((out, kern))
+    return outs
+
+
+def _bits(t):
+    return t.view(torch.int32) if t.dtype == torch.float32 else \
+        t.view(torch.int16) if t.dtype == torch.bfloat16 else t
+
+
+def _same(a, b):
+    # bit patterns, so that the NaN of a dropped token's log-probability compares equal
+    for k in ("stats", "logp", "logp_old", "flags", "dlogits"):
+        if a.get(k) is not None or b.get(k) is not None:
+            assert torch.equal(_bits(a[k]), _bits(b[k])), k
+
+
+@pytest.mark.parametrize("T", [1, 3, 300, 1500])
+def test_tmem_tier_equals_plain_kernel(T):
+    # fewer rows than CTAs, a few rounds of the row counter, and many
+    b = make_loss_batch("agentic_bf16_v151936", T=T, seed=T, device="cuda")
+    (tm, ktm), (pl, kpl) = _both(b)
+    assert ktm == "k2_fused_l2/tmem" and kpl == "k2_fused_l2"
+    _same(tm, pl)
+
+
+@pytest.mark.parametrize("variant", ["f32_logits", "f32_dlogits", "forward_only", "in_place",
+                                     "bad_ids_and_masked"])
+def test_tmem_tier_variants(variant):
+    name = "tight_f32_v151936" if variant == "f32_logits" else "agentic_bf16_v151936"
+    b = make_loss_batch(name, T=96, seed=11, device="cuda")
+    kw = {}
+    if variant == "f32_dlogits":
+        kw = dict(dlogits_f32=True)
+    elif variant == "forward_only":
+        kw = dict(dlogits=None)
+    elif variant == "bad_ids_and_masked":
+        b.ids[3] = -1
+        b.ids[40] = b.V
+        b.mask[10:30] = 0
+    if variant == "in_place":
+        outs = []
+        for tm in (1, 0):
+            z = b.z_theta.clone()
+            with occ.options(fused_tmem=tm):
+                out = occ.occ_decoupled_loss_fused(z, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                                   dlogits="inplace", **b.thresholds())
+                kern = occ.occ_last_kernel()
+            torch.cuda.synchronize()
+            outs.append((out, kern, z))
+        assert outs[0][1] == "k2_fused_l2/tmem" and outs[1][1] == "k2_fused_l2"
+        assert torch.equal(outs[0][2], outs[1][2])
+        _same(outs[0][0], outs[1][0])
+        return
+    (tm, ktm), (pl, kpl) = _both(b, **kw)
+    assert ktm == "k2_fused_l2/tmem" and kpl == "k2_fused_l2"
+    _same(tm, pl)
+    if variant == "bad_ids_and_masked":
+        st = occ.decode_loss_stats(tm["stats"])
+        m = b.mask.bool()
+        m[3] = m[40] = False
+        assert st.err == occ.DATA_ERR_BAD_ID and st.n_valid == int(m.sum())
+
+
+@pytest.mark.parametrize("V", [98304, 114688, 114696])
+def test_tmem_tier_threshold(V):
+    # 98304 bf16 rows (192 KB) hold 24 blocks in whole rounds: the plain kernel;
+    # 114688 hold 28 (the tier); 114696 one vector more (the walk's last round)
+    b = make_loss_batch("agentic_bf16_v151936", T=40, V=V, seed=V, device="cuda")
+    (tm, ktm), (pl, kpl) = _both(b)
+    assert ktm == expected_kernel("fused", V, 2, diag=False) and kpl == "k2_fused_l2"
+    assert ktm == ("k2_fused_l2" if V == 98304 else "k2_fused_l2/tmem")
+    _same(tm, pl)
+
+
+def test_diagnostics_and_head_option_keep_the_plain_kernel():
+    b = make_loss_batch("agentic_bf16_v151936", T=16, seed=2, device="cuda")
+    occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                 want_diagnostics=True, **b.thresholds())
+    assert occ.occ_last_kernel() == "k2_fused_l2"
+    with occ.options(fused_head_bytes=65536):
+        occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                     **b.thresholds())
+        assert occ.occ_last_kernel() == "k2_fused_l2"
+    torch.cuda.synchronize()
