@@ -370,7 +370,8 @@ typedef enum {
   OCC_OPT_FUSED_THREADS = 5,   /* threads per occ_decoupled_loss_fused CTA: 128, 256, 512 */
   OCC_OPT_FUSED_HEAD_BYTES = 6, /* its shared-memory head, bytes                       */
   OCC_OPT_FUSED_TMEM = 7,      /* 0: no tensor-memory row cache for long rows; 1: allowed */
-  OCC_OPT_COUNT_ = 8
+  OCC_OPT_K2_TMEM = 8,         /* the same for occ_decoupled_loss_fwd_bwd              */
+  OCC_OPT_COUNT_ = 9
 } occ_option;
 occ_status occ_set_option(occ_option opt, int64_t value);
 int64_t occ_get_option(occ_option opt);

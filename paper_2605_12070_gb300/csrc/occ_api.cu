@@ -51,7 +51,8 @@ static bool option_value_ok(occ_option opt, int64_t v) {
   if (v == -1) return true;
   switch (opt) {
     case OCC_OPT_K1_WARP:
-    case OCC_OPT_FUSED_TMEM: return v == 0 || v == 1;
+    case OCC_OPT_FUSED_TMEM:
+    case OCC_OPT_K2_TMEM: return v == 0 || v == 1;
     case OCC_OPT_K1_THREADS:
     case OCC_OPT_K2_THREADS:
     case OCC_OPT_FUSED_THREADS: return v == 128 || v == 256 || v == 512;

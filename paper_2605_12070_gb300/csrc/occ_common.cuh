@@ -216,6 +216,26 @@ __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// The tensor-memory tier of the loss kernels (512-thread CTAs, two per SM): a
+// row walks in blocks of 512 vectors; blocks [0, kTmHeadBlocks) go to the
+// shared-memory head (72 KB), blocks [kTmHeadBlocks, kTmHeadBlocks + kTmBlocks)
+// to tensor memory (128 KB: 256 columns of the 128 lanes, so two CTAs take the
+// SM's 512 columns), the rest is re-read from L2.  Thread t of warp w keeps
+// its vector of block k in lane 32 (w % 4) + t % 32, columns 64 (w / 4) + 4 k
+// to + 3.  The launchers take this tier only for rows whose tensor-memory
+// blocks lie in whole rounds of the walk (every thread loads its vector of
+// each such block, so the accesses stay warp-converged).
+constexpr int kTmThreads = 512;
+constexpr int kTmHeadBlocks = 9;
+constexpr int kTmBlocks = 16;
+constexpr uint32_t kTmCols = 256;
+
+// This warp's part of the CTA's tensor memory (base from tcgen05.alloc).
+__device__ __forceinline__ uint32_t tmem_warp_base(uint32_t base) {
+  const uint32_t w = threadIdx.x >> 5;
+  return base + ((32u * (w & 3u)) << 16) + (w >> 2) * 64u;
+}
+
 // ------------------------------------------------------------ row streaming
 
 // How a thread walks the vectors i = t, t + NT, t + 2 NT, ... < n of a row,

@@ -25,16 +25,6 @@
 
 namespace occ {
 
-// The tensor-memory tier (TM): rows walk in blocks of NT = 512 vectors; blocks
-// [0, kTmHeadBlocks) go to the shared-memory head (72 KB), blocks
-// [kTmHeadBlocks, kTmHeadBlocks + kTmBlocks) to tensor memory (128 KB: 256
-// columns of the 128 lanes, two CTAs per SM take the 512 columns), the rest is
-// re-read from L2.  The launcher takes this tier only for rows whose tensor-
-// memory blocks lie in full rounds of the walk.
-constexpr int kTmHeadBlocks = 9;
-constexpr int kTmBlocks = 16;
-constexpr uint32_t kTmCols = 256;
-
 // One 16-byte vector of the current row and the old row.
 struct RowPair {
   uint4 t, o;
@@ -46,6 +36,7 @@ struct RowPair {
 // have the same byte offset (checked on the host).
 template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
+  static_assert(!TM || (NT == kTmThreads && !PEEL), "the tensor-memory tier: 512 threads, aligned");
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ FusedRed red;
@@ -68,10 +59,6 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
     __syncthreads();
     tmem_fence_after_sync();
   }
-  // TM: this warp's tensor memory, its quarter of the lanes and 64 of the columns
-  auto tmem_warp = [&]() {
-    return tmem_sm + ((uint32_t)(32 * ((tid >> 5) & 3)) << 16) + (uint32_t)((tid >> 5) >> 2) * 64u;
-  };
   for (int64_t row_i = a.row0 + blockIdx.x;; row_i += gridDim.x) {
     int64_t row = row_i;
     if constexpr (TM) {  // rows from a counter that K0 cleared: no tail of unequal CTAs
@@ -147,7 +134,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
             const int k = j / NT - kTmHeadBlocks;
             if (k >= 0 && k < kTmBlocks) {
               __syncwarp();
-              tmem_st16(tmem_warp() + 4u * (uint32_t)k, r.t);
+              tmem_st16(tmem_warp_base(tmem_sm) + 4u * (uint32_t)k, r.t);
             }
           }
           consume(j, r.t, r.o);
@@ -206,7 +193,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
             [&](int j, const uint4& r) { emit(rb + j, r); });
         if constexpr (TM) {
           __syncwarp();
-          const uint32_t tw = tmem_warp();
+          const uint32_t tw = tmem_warp_base(tmem_sm);
           for (int k = 0; k < kTmBlocks; ++k) {
             const uint4 r = tmem_ld16(tw + 4u * (uint32_t)k);
             tmem_wait_ld();

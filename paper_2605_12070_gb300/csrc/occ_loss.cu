@@ -40,18 +40,42 @@ namespace occ {
 // sees the logits once and dlogits once.  Oldest-first bounds the time a line
 // waits in L2 by the longer of the two passes (newest-first lets the first
 // lines wait through both).  dlogits are written evict-first.
-template <typename Tin, typename Tout, int NT, int U, bool PEEL>
+//
+// TM (long aligned rows, 512 threads): the tensor-memory tier of
+// occ_common.cuh keeps 128 KB more of the row on chip, and the kernel runs
+// persistent, two CTAs per SM fetching rows from the workspace's counter.
+template <typename Tin, typename Tout, int NT, int U, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
+  static_assert(!TM || (NT == kTmThreads && !PEEL), "the tensor-memory tier: 512 threads, aligned");
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ RedScratch red;
   __shared__ float bc_g, bc_cb;
+  __shared__ uint32_t tmem_sm;  // TM: the CTA's tensor-memory address
+  __shared__ long long row_sm;  // TM: the row fetched for the CTA
   const uint64_t keep = l2_policy_evict_last();
   const uint64_t last = l2_policy_evict_first();
   const int tid = threadIdx.x;
   const int64_t V = a.V;
   const long long N = a.kp.denom > 0 ? a.kp.denom : *a.ws_N;
-  for (int64_t row = a.row0 + blockIdx.x; row < a.T; row += gridDim.x) {
+  if constexpr (TM) {
+    if (tid < 32) {
+      __syncwarp();
+      tmem_alloc(&tmem_sm, kTmCols);
+    }
+    tmem_fence_before_sync();
+    __syncthreads();
+    tmem_fence_after_sync();
+  }
+  for (int64_t row_i = a.row0 + blockIdx.x;; row_i += gridDim.x) {
+    int64_t row = row_i;
+    if constexpr (TM) {
+      __syncthreads();
+      if (tid == 0) row_sm = (long long)atomicAdd(a.ws_rows, 1u) + a.row0;
+      __syncthreads();
+      row = row_sm;
+    }
+    if (row >= a.T) break;
     const int id = a.ids[row];
     const bool m = (a.mask == nullptr) || (a.mask[row] != 0);
     const bool id_ok = id >= 0 && (int64_t)id < V;
@@ -99,10 +123,21 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
         tid, (int)nvec, [&](int j) { return ld_hint_v4(zv + j, keep); },
         [&](int j, const uint4& r) {
           if (j < nh) head_sm[j] = r;
+          if constexpr (TM) {  // block k of the tensor-memory part: the same for the whole CTA
+            const int k = j / NT - kTmHeadBlocks;
+            if (k >= 0 && k < kTmBlocks) {
+              __syncwarp();
+              tmem_st16(tmem_warp_base(tmem_sm) + 4u * (uint32_t)k, r);
+            }
+          }
           float x[VEC];
           Elem<Tin>::unpack(r, x);
           acc_add_fast(acc, x);
         });
+    if constexpr (TM) {
+      __syncwarp();
+      tmem_wait_st();
+    }
     float xt = 0.f, xp = 0.f;
     if ((int64_t)tid < ntail) {
       xt = Elem<Tin>::load(z + tail0 + tid);
@@ -150,12 +185,22 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
           }
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
-        // re-read part, oldest first: vectors head+tid, head+tid+NT, ... < nvec
-        const int64_t nre = nvec - head;
-        const uint4* zr = zv + head;
+        // re-read part, oldest first: vectors rb+tid, rb+tid+NT, ... < nvec
+        const int64_t rb = TM ? (int64_t)(kTmHeadBlocks + kTmBlocks) * NT : head;
+        const int64_t nre = nvec - rb;
+        const uint4* zr = zv + rb;
         walk_row<kW, U, NT>(
             tid, (int)nre, [&](int j) { return ld_hint_v4(zr + j, last); },
-            [&](int j, const uint4& r) { emit(head + j, r); });
+            [&](int j, const uint4& r) { emit(rb + j, r); });
+        if constexpr (TM) {
+          __syncwarp();
+          const uint32_t tw = tmem_warp_base(tmem_sm);
+          for (int k = 0; k < kTmBlocks; ++k) {
+            const uint4 r = tmem_ld16(tw + 4u * (uint32_t)k);
+            tmem_wait_ld();
+            emit((int64_t)(kTmHeadBlocks + k) * NT + tid, r);
+          }
+        }
         // on-chip head
 #pragma unroll 4
         for (int64_t j = tid; j < head; j += NT) emit(j, head_sm[j]);
@@ -172,6 +217,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
       }
     }
     __syncthreads();
+  }
+  if constexpr (TM) {
+    tmem_fence_before_sync();
+    __syncthreads();
+    tmem_fence_after_sync();
+    if (tid < 32) {
+      __syncwarp();
+      tmem_dealloc(tmem_sm, kTmCols);
+    }
   }
 }
 
@@ -296,7 +350,23 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     const size_t head_auto = nt_auto == 128   ? 16 * 1024
                              : nt_auto == 256 ? 0
                                               : two_cta_smem_budget((const void*)kern);
-    const size_t head_bytes = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
+    size_t head_bytes = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
+    // Long aligned rows take the tensor-memory tier when every tensor-memory block
+    // lies in whole rounds of the walk (8 blocks per round); OCC_OPT_K2_TMEM = 0 or
+    // a shape option keeps the plain kernel.
+    bool tm = false;
+    const int64_t step = 0x7fffffffLL;
+    const int64_t full_blocks = (int64_t)(a.V / Elem<Tin>::kVec) / (8 * kTmThreads) * 8;
+    if (vec && nt == kTmThreads && option(OCC_OPT_K2_TMEM) != 0 && head_opt < 0 && unroll < 0 &&
+        T < step && full_blocks >= kTmHeadBlocks + kTmBlocks) {
+      K2Kern kt = k2_loss_l2<Tin, Tout, kTmThreads, 8, false, true>;
+      const size_t tm_head = (size_t)kTmHeadBlocks * kTmThreads * 16;
+      if (two_cta_smem_budget((const void*)kt) >= tm_head) {
+        kern = kt;
+        head_bytes = tm_head;
+        tm = true;
+      }
+    }
     a.stage_bytes = (int64_t)head_bytes;
     if (head_bytes > 0) {
       cudaError_t e =
@@ -305,12 +375,16 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
         return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head_bytes,
                     cudaGetErrorString(e));
     }
-    note_kernel(peel ? "k2_loss_l2/peel" : "k2_loss_l2");
-    const int64_t step = 0x7fffffffLL;
-    for (int64_t r0 = 0; r0 < T; r0 += step) {
-      a.row0 = r0;
-      const unsigned grid = (unsigned)std::min<int64_t>(step, T - r0);
-      kern<<<grid, nt, head_bytes, s>>>(a);
+    note_kernel(tm ? "k2_loss_l2/tmem" : peel ? "k2_loss_l2/peel" : "k2_loss_l2");
+    if (tm) {  // persistent: two CTAs per SM (the register limit), rows from the counter
+      a.row0 = 0;
+      kern<<<(unsigned)std::min<int64_t>(T, (int64_t)sm_count() * 2), nt, head_bytes, s>>>(a);
+    } else {
+      for (int64_t r0 = 0; r0 < T; r0 += step) {
+        a.row0 = r0;
+        const unsigned grid = (unsigned)std::min<int64_t>(step, T - r0);
+        kern<<<grid, nt, head_bytes, s>>>(a);
+      }
     }
     return check_launch("occ_decoupled_loss_fwd_bwd");
   }

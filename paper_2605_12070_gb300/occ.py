@@ -42,7 +42,8 @@ EXPORTS = ("occ_token_logprob", "occ_loss_workspace_bytes", "occ_decoupled_loss_
 
 # occ_option codes (include/occ.h)
 OPTIONS = {"k1_warp": 0, "k1_threads": 1, "k2_threads": 2, "k2_head_bytes": 3, "k2_unroll": 4,
-           "fused_threads": 5, "fused_head_bytes": 6, "fused_tmem": 7}
+           "fused_threads": 5, "fused_head_bytes": 6, "fused_tmem": 7,
+           "k2_tmem": 8}
 
 
 class OccError(RuntimeError):

@@ -3,9 +3,10 @@
 the vector kernel when rows start on 16-byte boundaries, the peeled vector
 kernel when they do not but a row holds at least 16 vectors, else the
 element-load kernel; for K1, rows of up to 32 KB run one warp per row.  The
-fused kernel without diagnostics runs its tensor-memory tier on aligned rows of
-the 512-thread tier (over 112 KB) that hold at least 25 blocks of 512 vectors
-in whole rounds of 4 blocks."""
+fused kernel without diagnostics and K2 run their tensor-memory tiers on
+aligned rows of the 512-thread tier (over 112 KB) that hold at least 25 blocks
+of 512 vectors in whole rounds of the walk (4 blocks per round in the fused
+kernel, 8 in K2)."""
 
 
 def expected_kernel(kind, V, elem_size, diag=True):
@@ -19,6 +20,8 @@ def expected_kernel(kind, V, elem_size, diag=True):
     if (V * elem_size) % 16 == 0:
         nvec = V // vec
         if kind == "fused" and not diag and nvec * 16 > 112 * 1024 and nvec // 2048 * 4 >= 25:
+            return first + "/tmem"
+        if kind == "k2" and nvec * 16 > 112 * 1024 and nvec // 4096 * 8 >= 25:
             return first + "/tmem"
         return first
     return first + "/peel" if V >= 16 * vec else names[1]

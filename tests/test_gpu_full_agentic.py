@@ -167,7 +167,7 @@ def test_two_call_every_token(agentic):
     out = occ.occ_decoupled_loss_fwd_bwd(b.z_theta, b.ids, lp_old_gpu, b.logp_mu, b.adv, b.mask,
                                          **b.thresholds())
     torch.cuda.synchronize()
-    assert occ.occ_last_kernel() == "k2_loss_l2"
+    assert occ.occ_last_kernel() == "k2_loss_l2/tmem"   # the tensor-memory tier
     glo = lp_old_gpu.cpu().numpy().astype(np.float64)
     # K1 reads every row, masked or not: R1 on all 65536 rows
     assert np.abs(glo - lo64).max() <= LOGP_TIGHT

@@ -1,12 +1,13 @@
-"""The fused kernel's tensor-memory tier against its plain kernel, bit for bit.
+"""The tensor-memory tiers of the fused kernel and of K2 against their plain
+kernels, bit for bit.
 
-Long aligned rows without diagnostics keep 128 KB of the current row in tensor
-memory instead of re-reading it from L2, and the kernel runs persistent with
-rows fetched from a counter.  The arithmetic is the plain kernel's in the same
-order, so every output must equal the plain kernel's (OCC_OPT_FUSED_TMEM = 0)
-bit for bit: dlogits, the statistics, log pi_theta, log pi_old and the flags.
-The oracle comparisons of the default path (test_gpu_fused.py,
-test_gpu_full_agentic.py) run this tier on the long-row batches.
+Long aligned rows keep 128 KB of the current row in tensor memory instead of
+re-reading it from L2, and the kernel runs persistent with rows fetched from a
+counter.  The arithmetic is the plain kernel's in the same order, so every
+output must equal the plain kernel's (OCC_OPT_FUSED_TMEM / OCC_OPT_K2_TMEM = 0)
+bit for bit: dlogits, the statistics, the log-probabilities and the flags.  The
+oracle comparisons of the default paths (test_gpu_fused.py, test_gpu_loss.py,
+test_gpu_full_agentic.py) run these tiers on the long-row batches.
 """
 
 import pytest
@@ -111,3 +112,50 @@ def test_diagnostics_and_head_option_keep_the_plain_kernel():
                                      **b.thresholds())
         assert occ.occ_last_kernel() == "k2_fused_l2"
     torch.cuda.synchronize()
+
+
+def _k2_both(b, lp_old, **kw):
+    outs = []
+    for tm in (1, 0):
+        with occ.options(k2_tmem=tm):
+            out = occ.occ_decoupled_loss_fwd_bwd(b.z_theta, b.ids, lp_old, b.logp_mu, b.adv, b.mask,
+                                                 **b.thresholds(), **kw)
+            kern = occ.occ_last_kernel()
+        torch.cuda.synchronize()
+        outs.append((out, kern))
+    return outs
+
+
+@pytest.mark.parametrize("variant", ["plain", "few_rows", "many_rows", "f32_logits", "f32_dlogits",
+                                     "forward_only", "bad_ids_and_masked", "proxy"])
+def test_k2_tmem_tier_equals_plain_kernel(variant):
+    name = "tight_f32_v151936" if variant == "f32_logits" else "agentic_bf16_v151936"
+    T = {"few_rows": 3, "many_rows": 1500}.get(variant, 96)
+    b = make_loss_batch(name, T=T, seed=13, device="cuda")
+    lp_old, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    kw = {}
+    if variant == "f32_dlogits":
+        kw = dict(dlogits_f32=True)
+    elif variant == "forward_only":
+        kw = dict(dlogits=None)
+    elif variant == "proxy":
+        kw = dict(proxy="arithmetic", alpha=0.5)
+    elif variant == "bad_ids_and_masked":
+        b.ids[3] = -1
+        b.mask[10:30] = 0
+    (tm, ktm), (pl, kpl) = _k2_both(b, lp_old, **kw)
+    assert ktm == "k2_loss_l2/tmem" and kpl == "k2_loss_l2"
+    _same(tm, pl)
+
+
+@pytest.mark.parametrize("V", [131064, 131072, 131080])
+def test_k2_tmem_tier_threshold(V):
+    # K2 walks 8 blocks per round: 131064 bf16 rows (16383 vectors) hold 24 blocks
+    # in whole rounds (the plain kernel), 131072 hold 32 (the tier), 131080 one
+    # vector more
+    b = make_loss_batch("agentic_bf16_v151936", T=24, V=V, seed=V, device="cuda")
+    lp_old, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    (tm, ktm), (pl, kpl) = _k2_both(b, lp_old)
+    assert ktm == expected_kernel("k2", V, 2) and kpl == "k2_loss_l2"
+    assert ktm == ("k2_loss_l2" if V == 131064 else "k2_loss_l2/tmem")
+    _same(tm, pl)
