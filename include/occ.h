@@ -37,6 +37,15 @@
  *     V >= 128 (bf16) / 64 (f32); any other layout runs on a scalar-load
  *     kernel.  All three meet the same accuracy bounds; occ_last_kernel()
  *     names the one a call took.
+ *   - Long aligned rows of occ_decoupled_loss_fwd_bwd and
+ *     occ_decoupled_loss_fused (512-thread CTAs, rows of at least 25 blocks
+ *     of 512 16-byte vectors in whole rounds of the row walk; the fused call
+ *     without entropy or KL outputs) keep 128 KB of each current-logits row in
+ *     tensor memory: each CTA allocates 256 columns (tcgen05.alloc), two CTAs
+ *     per SM, so such a kernel holds all 512 columns of the SMs it runs on
+ *     until it ends.  A kernel of another stream that allocates tensor memory
+ *     on the same SM waits for it.  The results are bit for bit those of the
+ *     plain kernel (OCC_OPT_FUSED_TMEM / OCC_OPT_K2_TMEM = 0).
  */
 #ifndef OCC_H_
 #define OCC_H_
@@ -385,12 +394,12 @@ const char* occ_last_error(void);
 /* The row kernel that the last call on this host thread launched, as a static
  * string: "k1_logprob_warp", "k1_logprob_warp/peel", "k1_logprob_vec",
  * "k1_logprob_vec/peel", "k1_logprob_scalar",
- * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_stream", "k2_fused_l2",
- * "k2_fused_l2/peel", "k2_fused_stream",
- * "k2_fused_ring", "k3_ewma_vec", "k3_ewma_scalar", "k3_ewma_bf16" ("" when
- * the call launched none, e.g. T = 0 or an invalid argument).  "/peel" marks
- * the vector kernel run on rows that start off a 16-byte boundary.  Never
- * freed; valid until the next call on the thread. */
+ * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_l2/tmem", "k2_loss_stream",
+ * "k2_fused_l2", "k2_fused_l2/peel", "k2_fused_l2/tmem", "k2_fused_stream",
+ * "k3_ewma_vec", "k3_ewma_scalar", "k3_ewma_bf16" ("" when the call launched
+ * none, e.g. T = 0 or an invalid argument).  "/peel" marks the vector kernel
+ * run on rows that start off a 16-byte boundary, "/tmem" its tensor-memory
+ * tier.  Never freed; valid until the next call on the thread. */
 const char* occ_last_kernel(void);
 
 /* OCC_VERSION of the built library. */
