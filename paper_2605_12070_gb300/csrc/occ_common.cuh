@@ -216,19 +216,23 @@ __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// The tensor-memory tier of the loss kernels (512-thread CTAs, two per SM): a
-// row walks in blocks of 512 vectors; blocks [0, kTmHeadBlocks) go to the
-// shared-memory head (72 KB), blocks [kTmHeadBlocks, kTmHeadBlocks + kTmBlocks)
-// to tensor memory (128 KB: 256 columns of the 128 lanes, so two CTAs take the
-// SM's 512 columns), the rest is re-read from L2.  Thread t of warp w keeps
-// its vector of block k in lane 32 (w % 4) + t % 32, columns 64 (w / 4) + 4 k
-// to + 3.  The launchers take this tier only for rows whose tensor-memory
-// blocks lie in whole rounds of the walk (every thread loads its vector of
-// each such block, so the accesses stay warp-converged).
+// The tensor-memory tier of the loss kernels.  A row walks in blocks of NT
+// vectors (one per thread); after a shared-memory head of some blocks, the next
+// kTmBlocks blocks go to tensor memory and the rest is re-read from L2.  Each
+// thread keeps its kTmBlocks vectors in 4 kTmBlocks = 64 columns of its own
+// lane; warp w uses the lane quarter w % 4 and columns 64 floor(w / 4) on, so
+// a CTA takes NT / 2 columns: 256 for 512 threads (two CTAs per SM), 64 for 128
+// threads (eight per SM): the SM's 512 columns either way.  The launchers take
+// this tier only for rows whose tensor-memory blocks lie in whole rounds of the
+// walk (every thread loads its vector of each such block, so the accesses stay
+// warp-converged).
 constexpr int kTmThreads = 512;
-constexpr int kTmHeadBlocks = 9;
+constexpr int kTmHeadBlocks = 9;  // the 512-thread tier's head: 9 blocks of 512 vectors (72 KB)
 constexpr int kTmBlocks = 16;
-constexpr uint32_t kTmCols = 256;
+template <int NT>
+constexpr uint32_t tm_cols() {
+  return (uint32_t)NT / 2;
+}
 
 // This warp's part of the CTA's tensor memory (base from tcgen05.alloc).
 __device__ __forceinline__ uint32_t tmem_warp_base(uint32_t base) {

@@ -36,7 +36,9 @@ struct RowPair {
 // have the same byte offset (checked on the host).
 template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
-  static_assert(!TM || (NT == kTmThreads && !PEEL), "the tensor-memory tier: 512 threads, aligned");
+  static_assert(!TM || ((NT == kTmThreads || NT == 128) && !PEEL), "the tensor-memory tier");
+  // head blocks before the tensor-memory part: 72 KB at 512 threads, none at 128 (the plain kernel has none there either)
+  constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : 0;
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ FusedRed red;
@@ -53,7 +55,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
   if constexpr (TM) {
     if (tid < 32) {
       __syncwarp();
-      tmem_alloc(&tmem_sm, kTmCols);
+      tmem_alloc(&tmem_sm, tm_cols<NT>());
     }
     tmem_fence_before_sync();
     __syncthreads();
@@ -131,7 +133,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
         [&](int j) { return RowPair{ld_hint_v4(zv + j, keep), ld_hint_v4(zov + j, last)}; },
         [&](int j, const RowPair& r) {
           if constexpr (TM) {  // block k of the tensor-memory part: the same for the whole CTA
-            const int k = j / NT - kTmHeadBlocks;
+            const int k = j / NT - kHB;
             if (k >= 0 && k < kTmBlocks) {
               __syncwarp();
               tmem_st16(tmem_warp_base(tmem_sm) + 4u * (uint32_t)k, r.t);
@@ -185,7 +187,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
           }
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
-        const int64_t rb = TM ? (int64_t)(kTmHeadBlocks + kTmBlocks) * NT : head;  // first re-read
+        const int64_t rb = TM ? (int64_t)(kHB + kTmBlocks) * NT : head;  // first re-read
         const int64_t nre = nvec - rb;
         const uint4* zr = zv + rb;
         walk_row<kW, 8, NT>(  // 8 vectors in flight, whatever the forward pass's U
@@ -197,7 +199,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
           for (int k = 0; k < kTmBlocks; ++k) {
             const uint4 r = tmem_ld16(tw + 4u * (uint32_t)k);
             tmem_wait_ld();
-            emit((int64_t)(kTmHeadBlocks + k) * NT + tid, r);
+            emit((int64_t)(kHB + k) * NT + tid, r);
           }
         }
 #pragma unroll 4
@@ -222,7 +224,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) 
     tmem_fence_after_sync();
     if (tid < 32) {
       __syncwarp();
-      tmem_dealloc(tmem_sm, kTmCols);
+      tmem_dealloc(tmem_sm, tm_cols<NT>());
     }
   }
 }
@@ -360,19 +362,23 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
     const size_t head_auto =
         nt_auto == kFusedThreads ? two_cta_smem_budget((const void*)kern) : 0;
     size_t head = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
-    // Long aligned rows without diagnostics take the tensor-memory tier (GB300, agentic
-    // batch V = 151936: 8.06 ms against 8.31 ms, the L2 re-read misses gone) when every
-    // tensor-memory block lies in full rounds of the walk; OCC_OPT_FUSED_TMEM = 0 or a
-    // head size from OCC_OPT_FUSED_HEAD_BYTES keeps the plain kernel.
+    // Aligned rows without diagnostics in the 512- and 128-thread tiers take the
+    // tensor-memory tier (GB300, agentic batch V = 151936: 8.06 ms against 8.31 ms, the
+    // L2 re-read misses gone) when every tensor-memory block lies in whole rounds of
+    // the walk; OCC_OPT_FUSED_TMEM = 0 or a shape option (OCC_OPT_FUSED_THREADS,
+    // OCC_OPT_FUSED_HEAD_BYTES) keeps the plain kernel.
     bool tm = false;
     if constexpr (!DIAG) {
-      const int64_t full_blocks = (f.a.V / Elem<Tin>::kVec) /
-                                  ((int64_t)kFusedUnroll * kFusedThreads) * kFusedUnroll;
-      if (vec && nt == kFusedThreads && option(OCC_OPT_FUSED_TMEM) != 0 && head_opt < 0 &&
-          T < step && full_blocks >= kTmHeadBlocks + kTmBlocks) {
-        FusedKern kt = k2_fused_l2<Tin, Tout, kFusedThreads, kFusedUnroll, false, false, true>;
-        const size_t tm_head = (size_t)kTmHeadBlocks * kFusedThreads * 16;
-        if (two_cta_smem_budget((const void*)kt) >= tm_head) {
+      const int hb = nt == kTmThreads ? kTmHeadBlocks : 0;
+      const int64_t full_blocks =
+          (f.a.V / Elem<Tin>::kVec) / ((int64_t)kFusedUnroll * nt) * kFusedUnroll;
+      if (vec && (nt == kTmThreads || nt == 128) && option(OCC_OPT_FUSED_TMEM) != 0 &&
+          nt_opt < 0 && head_opt < 0 && T < step && full_blocks >= hb + kTmBlocks) {
+        FusedKern kt = nt == kTmThreads
+                           ? k2_fused_l2<Tin, Tout, kTmThreads, kFusedUnroll, false, false, true>
+                           : k2_fused_l2<Tin, Tout, 128, kFusedUnroll, false, false, true>;
+        const size_t tm_head = (size_t)hb * nt * 16;
+        if (tm_head == 0 || two_cta_smem_budget((const void*)kt) >= tm_head) {
           kern = kt;
           head = tm_head;
           tm = true;
@@ -388,9 +394,9 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
                     cudaGetErrorString(e));
     }
     note_kernel(tm ? "k2_fused_l2/tmem" : peel ? "k2_fused_l2/peel" : "k2_fused_l2");
-    if (tm) {  // persistent: two CTAs per SM (the register limit), rows from the counter
+    if (tm) {  // persistent: 1024 / nt CTAs per SM (the register limit), rows from the counter
       f.a.row0 = 0;
-      const unsigned grid = (unsigned)std::min<int64_t>(T, (int64_t)sm_count() * 2);
+      const unsigned grid = (unsigned)std::min<int64_t>(T, (int64_t)sm_count() * (1024 / nt));
       kern<<<grid, nt, head, s>>>(f);
     } else {
       for (int64_t r0 = 0; r0 < T; r0 += step) {

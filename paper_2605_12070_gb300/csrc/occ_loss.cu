@@ -46,7 +46,9 @@ namespace occ {
 // persistent, two CTAs per SM fetching rows from the workspace's counter.
 template <typename Tin, typename Tout, int NT, int U, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
-  static_assert(!TM || (NT == kTmThreads && !PEEL), "the tensor-memory tier: 512 threads, aligned");
+  static_assert(!TM || ((NT == kTmThreads || NT == 128) && !PEEL), "the tensor-memory tier");
+  // head blocks before the tensor-memory part: 72 KB at 512 threads, 16 KB at 128 (as the plain kernel)
+  constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : 8;
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ RedScratch red;
@@ -61,7 +63,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   if constexpr (TM) {
     if (tid < 32) {
       __syncwarp();
-      tmem_alloc(&tmem_sm, kTmCols);
+      tmem_alloc(&tmem_sm, tm_cols<NT>());
     }
     tmem_fence_before_sync();
     __syncthreads();
@@ -124,7 +126,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
         [&](int j, const uint4& r) {
           if (j < nh) head_sm[j] = r;
           if constexpr (TM) {  // block k of the tensor-memory part: the same for the whole CTA
-            const int k = j / NT - kTmHeadBlocks;
+            const int k = j / NT - kHB;
             if (k >= 0 && k < kTmBlocks) {
               __syncwarp();
               tmem_st16(tmem_warp_base(tmem_sm) + 4u * (uint32_t)k, r);
@@ -186,7 +188,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
           OutVecHint<Tout, VEC>::store(drow + jj * VEC, d, last);
         };
         // re-read part, oldest first: vectors rb+tid, rb+tid+NT, ... < nvec
-        const int64_t rb = TM ? (int64_t)(kTmHeadBlocks + kTmBlocks) * NT : head;
+        const int64_t rb = TM ? (int64_t)(kHB + kTmBlocks) * NT : head;
         const int64_t nre = nvec - rb;
         const uint4* zr = zv + rb;
         walk_row<kW, U, NT>(
@@ -198,7 +200,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
           for (int k = 0; k < kTmBlocks; ++k) {
             const uint4 r = tmem_ld16(tw + 4u * (uint32_t)k);
             tmem_wait_ld();
-            emit((int64_t)(kTmHeadBlocks + k) * NT + tid, r);
+            emit((int64_t)(kHB + k) * NT + tid, r);
           }
         }
         // on-chip head
@@ -224,7 +226,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
     tmem_fence_after_sync();
     if (tid < 32) {
       __syncwarp();
-      tmem_dealloc(tmem_sm, kTmCols);
+      tmem_dealloc(tmem_sm, tm_cols<NT>());
     }
   }
 }
@@ -351,17 +353,19 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
                              : nt_auto == 256 ? 0
                                               : two_cta_smem_budget((const void*)kern);
     size_t head_bytes = std::min(head_opt >= 0 ? (size_t)head_opt : head_auto, row_bytes);
-    // Long aligned rows take the tensor-memory tier when every tensor-memory block
-    // lies in whole rounds of the walk (8 blocks per round); OCC_OPT_K2_TMEM = 0 or
-    // a shape option keeps the plain kernel.
+    // Aligned rows in the 512- and 128-thread tiers take the tensor-memory tier when
+    // every tensor-memory block lies in whole rounds of the walk (8 blocks per round);
+    // OCC_OPT_K2_TMEM = 0 or a shape option keeps the plain kernel.
     bool tm = false;
     const int64_t step = 0x7fffffffLL;
-    const int64_t full_blocks = (int64_t)(a.V / Elem<Tin>::kVec) / (8 * kTmThreads) * 8;
-    if (vec && nt == kTmThreads && option(OCC_OPT_K2_TMEM) != 0 && head_opt < 0 && unroll < 0 &&
-        T < step && full_blocks >= kTmHeadBlocks + kTmBlocks) {
-      K2Kern kt = k2_loss_l2<Tin, Tout, kTmThreads, 8, false, true>;
-      const size_t tm_head = (size_t)kTmHeadBlocks * kTmThreads * 16;
-      if (two_cta_smem_budget((const void*)kt) >= tm_head) {
+    const int hb = nt == kTmThreads ? kTmHeadBlocks : 8;
+    const int64_t full_blocks = (int64_t)(a.V / Elem<Tin>::kVec) / (8 * (int64_t)nt) * 8;
+    if (vec && (nt == kTmThreads || nt == 128) && option(OCC_OPT_K2_TMEM) != 0 && nt_opt < 0 &&
+        head_opt < 0 && unroll < 0 && T < step && full_blocks >= hb + kTmBlocks) {
+      K2Kern kt = nt == kTmThreads ? k2_loss_l2<Tin, Tout, kTmThreads, 8, false, true>
+                                   : k2_loss_l2<Tin, Tout, 128, 8, false, true>;
+      const size_t tm_head = (size_t)hb * nt * 16;
+      if (nt == 128 || two_cta_smem_budget((const void*)kt) >= tm_head) {
         kern = kt;
         head_bytes = tm_head;
         tm = true;
@@ -376,9 +380,10 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
                     cudaGetErrorString(e));
     }
     note_kernel(tm ? "k2_loss_l2/tmem" : peel ? "k2_loss_l2/peel" : "k2_loss_l2");
-    if (tm) {  // persistent: two CTAs per SM (the register limit), rows from the counter
+    if (tm) {  // persistent: 1024 / nt CTAs per SM (the register limit), rows from the counter
       a.row0 = 0;
-      kern<<<(unsigned)std::min<int64_t>(T, (int64_t)sm_count() * 2), nt, head_bytes, s>>>(a);
+      kern<<<(unsigned)std::min<int64_t>(T, (int64_t)sm_count() * (1024 / nt)), nt, head_bytes,
+             s>>>(a);
     } else {
       for (int64_t r0 = 0; r0 < T; r0 += step) {
         a.row0 = r0;

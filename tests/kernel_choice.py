@@ -4,9 +4,10 @@ the vector kernel when rows start on 16-byte boundaries, the peeled vector
 kernel when they do not but a row holds at least 16 vectors, else the
 element-load kernel; for K1, rows of up to 32 KB run one warp per row.  The
 fused kernel without diagnostics and K2 run their tensor-memory tiers on
-aligned rows of the 512-thread tier (over 112 KB) that hold at least 25 blocks
-of 512 vectors in whole rounds of the walk (4 blocks per round in the fused
-kernel, 8 in K2)."""
+aligned rows of the 512-thread tier (over 112 KB) and of the 128-thread tier
+(up to 64 KB) whose head and 16 tensor-memory blocks (of NT vectors) lie in
+whole rounds of the walk (4 blocks per round in the fused kernel, 8 in K2;
+heads of 9 blocks at 512 threads, of 0 / 8 blocks at 128)."""
 
 
 def expected_kernel(kind, V, elem_size, diag=True):
@@ -18,10 +19,13 @@ def expected_kernel(kind, V, elem_size, diag=True):
     if kind == "k1" and (V // vec) * 16 <= 32 * 1024:  # K1 rows up to 32 KB: one warp each
         first = "k1_logprob_warp"
     if (V * elem_size) % 16 == 0:
-        nvec = V // vec
-        if kind == "fused" and not diag and nvec * 16 > 112 * 1024 and nvec // 2048 * 4 >= 25:
+        nvec, rb = V // vec, (V // vec) * 16
+        if kind == "fused" and not diag and (
+                (rb > 112 * 1024 and nvec // 2048 * 4 >= 9 + 16) or
+                (rb <= 64 * 1024 and nvec // 512 * 4 >= 16)):
             return first + "/tmem"
-        if kind == "k2" and nvec * 16 > 112 * 1024 and nvec // 4096 * 8 >= 25:
+        if kind == "k2" and ((rb > 112 * 1024 and nvec // 4096 * 8 >= 9 + 16) or
+                             (rb <= 64 * 1024 and nvec // 1024 * 8 >= 8 + 16)):
             return first + "/tmem"
         return first
     return first + "/peel" if V >= 16 * vec else names[1]

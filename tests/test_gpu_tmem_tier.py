@@ -159,3 +159,20 @@ def test_k2_tmem_tier_threshold(V):
     assert ktm == expected_kernel("k2", V, 2) and kpl == "k2_loss_l2"
     assert ktm == ("k2_loss_l2" if V == 131064 else "k2_loss_l2/tmem")
     _same(tm, pl)
+
+
+@pytest.mark.parametrize("V,T", [(32000, 600), (32000, 2), (24000, 300), (16384, 100)])
+def test_short_row_tier_equals_plain_kernels(V, T):
+    # the 128-thread tier: 64 columns per CTA, eight CTAs per SM
+    name = "tiny_f32_v4096" if V == 16384 else "grpo_bf16_v32000"
+    b = make_loss_batch(name, T=T, V=V, seed=V + T, device="cuda")
+    es = b.z_theta.element_size()
+    (tm, ktm), (pl, kpl) = _both(b)
+    assert ktm == expected_kernel("fused", V, es, diag=False) == "k2_fused_l2/tmem"
+    assert kpl == "k2_fused_l2"
+    _same(tm, pl)
+    lp_old, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    (tm, ktm), (pl, kpl) = _k2_both(b, lp_old)
+    assert ktm == expected_kernel("k2", V, es) and kpl == "k2_loss_l2"
+    assert ktm == ("k2_loss_l2" if V == 24000 else "k2_loss_l2/tmem")
+    _same(tm, pl)
