@@ -37,15 +37,17 @@
  *     V >= 128 (bf16) / 64 (f32); any other layout runs on a scalar-load
  *     kernel.  All three meet the same accuracy bounds; occ_last_kernel()
  *     names the one a call took.
- *   - Long aligned rows of occ_decoupled_loss_fwd_bwd and
- *     occ_decoupled_loss_fused (512-thread CTAs, rows of at least 25 blocks
- *     of 512 16-byte vectors in whole rounds of the row walk; the fused call
- *     without entropy or KL outputs) keep 128 KB of each current-logits row in
- *     tensor memory: each CTA allocates 256 columns (tcgen05.alloc), two CTAs
- *     per SM, so such a kernel holds all 512 columns of the SMs it runs on
- *     until it ends.  A kernel of another stream that allocates tensor memory
- *     on the same SM waits for it.  The results are bit for bit those of the
- *     plain kernel (OCC_OPT_FUSED_TMEM / OCC_OPT_K2_TMEM = 0).
+ *   - Aligned rows of occ_decoupled_loss_fwd_bwd and occ_decoupled_loss_fused
+ *     (the fused call without entropy or KL outputs) keep part of each
+ *     current-logits row in tensor memory: rows over 112 KB hold 128 KB there
+ *     (512-thread CTAs allocating 256 columns each, two per SM), rows of up
+ *     to 64 KB hold 32 KB (128-thread CTAs, 64 columns, eight per SM), when
+ *     the row is long enough for the blocks to lie in whole rounds of the row
+ *     walk.  Such a kernel holds all 512 tensor-memory columns of the SMs it
+ *     runs on until it ends (tcgen05.alloc); a kernel of another stream that
+ *     allocates tensor memory on the same SM waits for it.  The results are
+ *     bit for bit those of the plain kernel (OCC_OPT_FUSED_TMEM /
+ *     OCC_OPT_K2_TMEM = 0).
  */
 #ifndef OCC_H_
 #define OCC_H_
