@@ -40,7 +40,8 @@
  *   - Aligned rows of occ_decoupled_loss_fwd_bwd and occ_decoupled_loss_fused
  *     (the fused call without entropy or KL outputs) keep part of each
  *     current-logits row in tensor memory: rows over 112 KB hold 128 KB there
- *     (512-thread CTAs allocating 256 columns each, two per SM), rows of up
+ *     (512-thread CTAs allocating 256 columns each, two per SM), rows of 64
+ *     to 112 KB hold 64 KB (256 threads, 128 columns, four per SM), rows of up
  *     to 64 KB hold 32 KB (128-thread CTAs, 64 columns, eight per SM), when
  *     the row is long enough for the blocks to lie in whole rounds of the row
  *     walk.  Such a kernel holds all 512 tensor-memory columns of the SMs it

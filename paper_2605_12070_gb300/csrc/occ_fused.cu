@@ -36,8 +36,10 @@ struct RowPair {
 // have the same byte offset (checked on the host).
 template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
-  static_assert(!TM || ((NT == kTmThreads || NT == 128) && !PEEL), "the tensor-memory tier");
-  // head blocks before the tensor-memory part: 72 KB at 512 threads, none at 128 (the plain kernel has none there either)
+  static_assert(!TM || ((NT == kTmThreads || NT == 256 || NT == 128) && !PEEL),
+                "the tensor-memory tier");
+  // head blocks before the tensor-memory part: 72 KB at 512 threads, none at 256 and 128 (the
+  // plain kernel has none there either)
   constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : 0;
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
@@ -372,11 +374,11 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
       const int hb = nt == kTmThreads ? kTmHeadBlocks : 0;
       const int64_t full_blocks =
           (f.a.V / Elem<Tin>::kVec) / ((int64_t)kFusedUnroll * nt) * kFusedUnroll;
-      if (vec && (nt == kTmThreads || nt == 128) && option(OCC_OPT_FUSED_TMEM) != 0 &&
+      if (vec && (nt == kTmThreads || nt == 256 || nt == 128) && option(OCC_OPT_FUSED_TMEM) != 0 &&
           nt_opt < 0 && head_opt < 0 && T < step && full_blocks >= hb + kTmBlocks) {
-        FusedKern kt = nt == kTmThreads
-                           ? k2_fused_l2<Tin, Tout, kTmThreads, kFusedUnroll, false, false, true>
-                           : k2_fused_l2<Tin, Tout, 128, kFusedUnroll, false, false, true>;
+        FusedKern kt = nt == kTmThreads ? k2_fused_l2<Tin, Tout, kTmThreads, kFusedUnroll, false, false, true>
+                       : nt == 256      ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, false, false, true>
+                                        : k2_fused_l2<Tin, Tout, 128, kFusedUnroll, false, false, true>;
         const size_t tm_head = (size_t)hb * nt * 16;
         if (tm_head == 0 || two_cta_smem_budget((const void*)kt) >= tm_head) {
           kern = kt;

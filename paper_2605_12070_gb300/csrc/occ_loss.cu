@@ -46,9 +46,11 @@ namespace occ {
 // persistent, two CTAs per SM fetching rows from the workspace's counter.
 template <typename Tin, typename Tout, int NT, int U, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
-  static_assert(!TM || ((NT == kTmThreads || NT == 128) && !PEEL), "the tensor-memory tier");
-  // head blocks before the tensor-memory part: 72 KB at 512 threads, 16 KB at 128 (as the plain kernel)
-  constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : 8;
+  static_assert(!TM || ((NT == kTmThreads || NT == 256 || NT == 128) && !PEEL),
+                "the tensor-memory tier");
+  // head blocks before the tensor-memory part: 72 KB at 512 threads, none at 256 and 16 KB at
+  // 128 (as the plain kernel)
+  constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : NT == 256 ? 0 : 8;
   constexpr int VEC = Elem<Tin>::kVec;
   extern __shared__ __align__(16) uint4 head_sm[];
   __shared__ RedScratch red;
@@ -358,14 +360,16 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     // OCC_OPT_K2_TMEM = 0 or a shape option keeps the plain kernel.
     bool tm = false;
     const int64_t step = 0x7fffffffLL;
-    const int hb = nt == kTmThreads ? kTmHeadBlocks : 8;
+    const int hb = nt == kTmThreads ? kTmHeadBlocks : nt == 256 ? 0 : 8;
     const int64_t full_blocks = (int64_t)(a.V / Elem<Tin>::kVec) / (8 * (int64_t)nt) * 8;
-    if (vec && (nt == kTmThreads || nt == 128) && option(OCC_OPT_K2_TMEM) != 0 && nt_opt < 0 &&
+    if (vec && (nt == kTmThreads || nt == 256 || nt == 128) && option(OCC_OPT_K2_TMEM) != 0 &&
+        nt_opt < 0 &&
         head_opt < 0 && unroll < 0 && T < step && full_blocks >= hb + kTmBlocks) {
       K2Kern kt = nt == kTmThreads ? k2_loss_l2<Tin, Tout, kTmThreads, 8, false, true>
+                  : nt == 256      ? k2_loss_l2<Tin, Tout, 256, 8, false, true>
                                    : k2_loss_l2<Tin, Tout, 128, 8, false, true>;
       const size_t tm_head = (size_t)hb * nt * 16;
-      if (nt == 128 || two_cta_smem_budget((const void*)kt) >= tm_head) {
+      if (nt != kTmThreads || two_cta_smem_budget((const void*)kt) >= tm_head) {
         kern = kt;
         head_bytes = tm_head;
         tm = true;

@@ -4,10 +4,10 @@ the vector kernel when rows start on 16-byte boundaries, the peeled vector
 kernel when they do not but a row holds at least 16 vectors, else the
 element-load kernel; for K1, rows of up to 32 KB run one warp per row.  The
 fused kernel without diagnostics and K2 run their tensor-memory tiers on
-aligned rows of the 512-thread tier (over 112 KB) and of the 128-thread tier
-(up to 64 KB) whose head and 16 tensor-memory blocks (of NT vectors) lie in
-whole rounds of the walk (4 blocks per round in the fused kernel, 8 in K2;
-heads of 9 blocks at 512 threads, of 0 / 8 blocks at 128)."""
+aligned rows (CTAs of 128 threads up to 64 KB rows, 256 up to 112 KB, 512
+beyond) whose head and 16 tensor-memory blocks (of NT vectors) lie in whole
+rounds of the walk (4 blocks per round in the fused kernel, 8 in K2; heads of 9
+blocks at 512 threads, none at 256, none / 8 blocks at 128)."""
 
 
 def expected_kernel(kind, V, elem_size, diag=True):
@@ -20,12 +20,14 @@ def expected_kernel(kind, V, elem_size, diag=True):
         first = "k1_logprob_warp"
     if (V * elem_size) % 16 == 0:
         nvec, rb = V // vec, (V // vec) * 16
-        if kind == "fused" and not diag and (
-                (rb > 112 * 1024 and nvec // 2048 * 4 >= 9 + 16) or
-                (rb <= 64 * 1024 and nvec // 512 * 4 >= 16)):
-            return first + "/tmem"
-        if kind == "k2" and ((rb > 112 * 1024 and nvec // 4096 * 8 >= 9 + 16) or
-                             (rb <= 64 * 1024 and nvec // 1024 * 8 >= 8 + 16)):
-            return first + "/tmem"
+        nt = 128 if rb <= 64 * 1024 else 256 if rb <= 112 * 1024 else 512
+        if kind == "fused" and not diag:
+            head = 9 if nt == 512 else 0
+            if nvec // (4 * nt) * 4 >= head + 16:
+                return first + "/tmem"
+        if kind == "k2":
+            head = {512: 9, 256: 0, 128: 8}[nt]
+            if nvec // (8 * nt) * 8 >= head + 16:
+                return first + "/tmem"
         return first
     return first + "/peel" if V >= 16 * vec else names[1]

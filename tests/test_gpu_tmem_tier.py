@@ -161,9 +161,11 @@ def test_k2_tmem_tier_threshold(V):
     _same(tm, pl)
 
 
-@pytest.mark.parametrize("V,T", [(32000, 600), (32000, 2), (24000, 300), (16384, 100)])
+@pytest.mark.parametrize("V,T", [(32000, 600), (32000, 2), (24000, 300), (16384, 100),
+                                 (50000, 300), (40000, 5)])
 def test_short_row_tier_equals_plain_kernels(V, T):
-    # the 128-thread tier: 64 columns per CTA, eight CTAs per SM
+    # the 128-thread tier (64 columns per CTA, eight CTAs per SM) and the 256-thread
+    # tier (128 columns, four per SM: V = 40000 and 50000 bf16)
     name = "tiny_f32_v4096" if V == 16384 else "grpo_bf16_v32000"
     b = make_loss_batch(name, T=T, V=V, seed=V + T, device="cuda")
     es = b.z_theta.element_size()
