@@ -37,8 +37,9 @@
  *     V >= 128 (bf16) / 64 (f32); any other layout runs on a scalar-load
  *     kernel.  All three meet the same accuracy bounds; occ_last_kernel()
  *     names the one a call took.
- *   - Aligned rows of occ_decoupled_loss_fwd_bwd and occ_decoupled_loss_fused
- *     (the fused call without entropy or KL outputs) keep part of each
+ *   - Rows of the vector kernels (aligned or peeled) of
+ *     occ_decoupled_loss_fwd_bwd and occ_decoupled_loss_fused (the fused call
+ *     without entropy or KL outputs) keep part of each
  *     current-logits row in tensor memory: rows over 112 KB hold 128 KB there
  *     (512-thread CTAs allocating 256 columns each, two per SM), rows of 64
  *     to 112 KB hold 64 KB (256 threads, 128 columns, four per SM), rows of up
@@ -400,9 +401,10 @@ const char* occ_last_error(void);
  * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_l2/tmem", "k2_loss_stream",
  * "k2_fused_l2", "k2_fused_l2/peel", "k2_fused_l2/tmem", "k2_fused_stream",
  * "k3_ewma_vec", "k3_ewma_scalar", "k3_ewma_bf16" ("" when the call launched
- * none, e.g. T = 0 or an invalid argument).  "/peel" marks the vector kernel
- * run on rows that start off a 16-byte boundary, "/tmem" its tensor-memory
- * tier.  Never freed; valid until the next call on the thread. */
+ * none, e.g. T = 0 or an invalid argument), and "k2_loss_l2/peel/tmem",
+ * "k2_fused_l2/peel/tmem".  "/peel" marks the vector kernel run on rows that
+ * start off a 16-byte boundary, "/tmem" its tensor-memory tier.  Never freed;
+ * valid until the next call on the thread. */
 const char* occ_last_kernel(void);
 
 /* OCC_VERSION of the built library. */

@@ -36,8 +36,7 @@ struct RowPair {
 // have the same byte offset (checked on the host).
 template <typename Tin, typename Tout, int NT, int U, bool DIAG, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_fused_l2(const FusedArgs f) {
-  static_assert(!TM || ((NT == kTmThreads || NT == 256 || NT == 128) && !PEEL),
-                "the tensor-memory tier");
+  static_assert(!TM || NT == kTmThreads || NT == 256 || NT == 128, "the tensor-memory tier");
   // head blocks before the tensor-memory part: 72 KB at 512 threads, none at 256 and 128 (the
   // plain kernel has none there either)
   constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : 0;
@@ -322,6 +321,14 @@ static FusedKern fused_kernel(int nt) {
                      : k2_fused_l2<Tin, Tout, kFusedThreads, U, DIAG, PEEL>;
 }
 
+// The tensor-memory tier's instantiation for a CTA size (4 row pairs in flight).
+template <typename Tin, typename Tout, bool PEEL>
+static FusedKern tm_kernel(int nt) {
+  return nt == kTmThreads ? k2_fused_l2<Tin, Tout, kTmThreads, kFusedUnroll, false, PEEL, true>
+         : nt == 256      ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, false, PEEL, true>
+                          : k2_fused_l2<Tin, Tout, 128, kFusedUnroll, false, PEEL, true>;
+}
+
 // Rows off a 16-byte boundary run the vector kernel peeled when the old-logits
 // and gradient rows sit at the same byte offsets as the current-logits rows
 // (same element size; base addresses and row strides congruent modulo 16
@@ -371,14 +378,16 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
     // OCC_OPT_FUSED_HEAD_BYTES) keeps the plain kernel.
     bool tm = false;
     if constexpr (!DIAG) {
+      // rows of a peeled call lose up to VEC - 1 elements to their scalar lead
       const int hb = nt == kTmThreads ? kTmHeadBlocks : 0;
-      const int64_t full_blocks =
-          (f.a.V / Elem<Tin>::kVec) / ((int64_t)kFusedUnroll * nt) * kFusedUnroll;
-      if (vec && (nt == kTmThreads || nt == 256 || nt == 128) && option(OCC_OPT_FUSED_TMEM) != 0 &&
-          nt_opt < 0 && head_opt < 0 && T < step && full_blocks >= hb + kTmBlocks) {
-        FusedKern kt = nt == kTmThreads ? k2_fused_l2<Tin, Tout, kTmThreads, kFusedUnroll, false, false, true>
-                       : nt == 256      ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, false, false, true>
-                                        : k2_fused_l2<Tin, Tout, 128, kFusedUnroll, false, false, true>;
+      const int64_t nvec_min = (f.a.V - (peel ? Elem<Tin>::kVec - 1 : 0)) / Elem<Tin>::kVec;
+      const int64_t full_blocks = nvec_min / ((int64_t)kFusedUnroll * nt) * kFusedUnroll;
+      if ((vec || peel) && (nt == kTmThreads || nt == 256 || nt == 128) &&
+          option(OCC_OPT_FUSED_TMEM) != 0 && nt_opt < 0 && head_opt < 0 && T < step &&
+          full_blocks >= hb + kTmBlocks) {
+        FusedKern kt = tm_kernel<Tin, Tout, false>(nt);
+        if constexpr (sizeof(Tin) == sizeof(Tout))
+          if (peel) kt = tm_kernel<Tin, Tout, true>(nt);
         const size_t tm_head = (size_t)hb * nt * 16;
         if (tm_head == 0 || two_cta_smem_budget((const void*)kt) >= tm_head) {
           kern = kt;
@@ -395,7 +404,8 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
         return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head,
                     cudaGetErrorString(e));
     }
-    note_kernel(tm ? "k2_fused_l2/tmem" : peel ? "k2_fused_l2/peel" : "k2_fused_l2");
+    note_kernel(tm ? (peel ? "k2_fused_l2/peel/tmem" : "k2_fused_l2/tmem")
+                   : peel ? "k2_fused_l2/peel" : "k2_fused_l2");
     if (tm) {  // persistent: 1024 / nt CTAs per SM (the register limit), rows from the counter
       f.a.row0 = 0;
       const unsigned grid = (unsigned)std::min<int64_t>(T, (int64_t)sm_count() * (1024 / nt));

@@ -46,8 +46,7 @@ namespace occ {
 // persistent, two CTAs per SM fetching rows from the workspace's counter.
 template <typename Tin, typename Tout, int NT, int U, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
-  static_assert(!TM || ((NT == kTmThreads || NT == 256 || NT == 128) && !PEEL),
-                "the tensor-memory tier");
+  static_assert(!TM || NT == kTmThreads || NT == 256 || NT == 128, "the tensor-memory tier");
   // head blocks before the tensor-memory part: 72 KB at 512 threads, none at 256 and 16 KB at
   // 128 (as the plain kernel)
   constexpr int kHB = NT == kTmThreads ? kTmHeadBlocks : NT == 256 ? 0 : 8;
@@ -317,6 +316,15 @@ static K2Kern l2_kernel(int nt, int unroll) {
                        : k2_loss_l2<Tin, Tout, 512, 8, PEEL>;
 }
 
+// The tensor-memory tier's instantiation for a CTA size: the plain kernel's
+// vectors in flight (6 for peeled 512-thread rows, else 8).
+template <typename Tin, typename Tout, bool PEEL>
+static K2Kern tm_kernel(int nt) {
+  return nt == kTmThreads ? k2_loss_l2<Tin, Tout, kTmThreads, PEEL ? 6 : 8, PEEL, true>
+         : nt == 256      ? k2_loss_l2<Tin, Tout, 256, 8, PEEL, true>
+                          : k2_loss_l2<Tin, Tout, 128, 8, PEEL, true>;
+}
+
 // Rows that are not 16-byte aligned can run the vector kernel peeled when the
 // gradient rows sit at the same byte offsets as the logits rows (same element
 // size, base addresses and row strides congruent modulo 16 bytes) and a row
@@ -361,13 +369,16 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
     bool tm = false;
     const int64_t step = 0x7fffffffLL;
     const int hb = nt == kTmThreads ? kTmHeadBlocks : nt == 256 ? 0 : 8;
-    const int64_t full_blocks = (int64_t)(a.V / Elem<Tin>::kVec) / (8 * (int64_t)nt) * 8;
-    if (vec && (nt == kTmThreads || nt == 256 || nt == 128) && option(OCC_OPT_K2_TMEM) != 0 &&
-        nt_opt < 0 &&
-        head_opt < 0 && unroll < 0 && T < step && full_blocks >= hb + kTmBlocks) {
-      K2Kern kt = nt == kTmThreads ? k2_loss_l2<Tin, Tout, kTmThreads, 8, false, true>
-                  : nt == 256      ? k2_loss_l2<Tin, Tout, 256, 8, false, true>
-                                   : k2_loss_l2<Tin, Tout, 128, 8, false, true>;
+    const int tu = (peel && nt == kTmThreads) ? 6 : 8;  // vectors in flight, as the plain kernel's
+    // rows of a peeled call lose up to VEC - 1 elements to their scalar lead
+    const int64_t nvec_min = (a.V - (peel ? Elem<Tin>::kVec - 1 : 0)) / Elem<Tin>::kVec;
+    const int64_t full_blocks = nvec_min / ((int64_t)tu * nt) * tu;
+    if ((vec || peel) && (nt == kTmThreads || nt == 256 || nt == 128) &&
+        option(OCC_OPT_K2_TMEM) != 0 && nt_opt < 0 && head_opt < 0 && unroll < 0 && T < step &&
+        full_blocks >= hb + kTmBlocks) {
+      K2Kern kt = tm_kernel<Tin, Tout, false>(nt);
+      if constexpr (sizeof(Tin) == sizeof(Tout))
+        if (peel) kt = tm_kernel<Tin, Tout, true>(nt);
       const size_t tm_head = (size_t)hb * nt * 16;
       if (nt != kTmThreads || two_cta_smem_budget((const void*)kt) >= tm_head) {
         kern = kt;
@@ -383,7 +394,8 @@ static occ_status launch_k2(K2Args a, bool vec, cudaStream_t s) {
         return fail(OCC_ERR_CUDA, "cudaFuncSetAttribute(smem=%zu): %s", head_bytes,
                     cudaGetErrorString(e));
     }
-    note_kernel(tm ? "k2_loss_l2/tmem" : peel ? "k2_loss_l2/peel" : "k2_loss_l2");
+    note_kernel(tm ? (peel ? "k2_loss_l2/peel/tmem" : "k2_loss_l2/tmem")
+                   : peel ? "k2_loss_l2/peel" : "k2_loss_l2");
     if (tm) {  // persistent: 1024 / nt CTAs per SM (the register limit), rows from the counter
       a.row0 = 0;
       kern<<<(unsigned)std::min<int64_t>(T, (int64_t)sm_count() * (1024 / nt)), nt, head_bytes,

@@ -10,6 +10,17 @@ rounds of the walk (4 blocks per round in the fused kernel, 8 in K2; heads of 9
 blocks at 512 threads, none at 256, none / 8 blocks at 128)."""
 
 
+def _tmem(kind, nvec, rb, diag, peel):
+    nt = 128 if rb <= 64 * 1024 else 256 if rb <= 112 * 1024 else 512
+    if kind == "fused" and not diag:
+        head, u = (9 if nt == 512 else 0), 4
+    elif kind == "k2":
+        head, u = {512: 9, 256: 0, 128: 8}[nt], (6 if peel and nt == 512 else 8)
+    else:
+        return False
+    return nvec // (u * nt) * u >= head + 16
+
+
 def expected_kernel(kind, V, elem_size, diag=True):
     vec = 16 // elem_size
     names = {"k1": ("k1_logprob_vec", "k1_logprob_scalar"),
@@ -18,16 +29,10 @@ def expected_kernel(kind, V, elem_size, diag=True):
     first = names[0]
     if kind == "k1" and (V // vec) * 16 <= 32 * 1024:  # K1 rows up to 32 KB: one warp each
         first = "k1_logprob_warp"
+    rb = (V // vec) * 16
     if (V * elem_size) % 16 == 0:
-        nvec, rb = V // vec, (V // vec) * 16
-        nt = 128 if rb <= 64 * 1024 else 256 if rb <= 112 * 1024 else 512
-        if kind == "fused" and not diag:
-            head = 9 if nt == 512 else 0
-            if nvec // (4 * nt) * 4 >= head + 16:
-                return first + "/tmem"
-        if kind == "k2":
-            head = {512: 9, 256: 0, 128: 8}[nt]
-            if nvec // (8 * nt) * 8 >= head + 16:
-                return first + "/tmem"
-        return first
-    return first + "/peel" if V >= 16 * vec else names[1]
+        return first + ("/tmem" if _tmem(kind, V // vec, rb, diag, False) else "")
+    if V < 16 * vec:
+        return names[1]
+    # peeled rows lose up to vec - 1 elements to their scalar lead
+    return first + "/peel" + ("/tmem" if _tmem(kind, (V - vec + 1) // vec, rb, diag, True) else "")

@@ -216,14 +216,16 @@ def test_fused_full_size_agentic_sampled():
 
 def test_fused_odd_vocab_past_2_31_logits_sampled():
     """An odd vocabulary (ld = V = 50257: rows off 16-byte boundaries, the
-    peeled kernel) over more than 2^31 logits per tensor, so row offsets pass
-    4 GB; sampled rows (the first, the last, random ones) against the oracle,
-    dlogits included."""
+    peeled kernel and its tensor-memory tier) over more than 2^31 logits per
+    tensor, so row offsets pass 4 GB; sampled rows (the first, the last, random
+    ones) against the oracle, dlogits included."""
     b = make_loss_batch("grpo_bf16_v32000", T=45_000, V=50_257, seed=6, device="cuda")
     T, V = b.T, b.V
     assert T * V > 2 ** 31
     out = _fused(b)
-    assert occ.occ_last_kernel() == "k2_fused_l2/peel"
+    # the peeled rows of the 256-thread tier keep 64 KB each in tensor memory
+    assert occ.occ_last_kernel() == expected_kernel("fused", V, 2, diag=False) == \
+        "k2_fused_l2/peel/tmem"
     mask = np.ones(T, np.uint8) if b.mask is None else b.mask.cpu().numpy()
     rng = np.random.default_rng(6)
     rows = np.unique(np.concatenate([rng.choice(T, 96, replace=False), [0, 1, T - 2, T - 1]]))

@@ -77,7 +77,8 @@ def test_k2_peeled_long_rows_every_unroll(unroll):
     with occ.options(**shape):
         out = occ.occ_decoupled_loss_fwd_bwd(z, ids, torch.from_numpy(fp32(lo64)).cuda(), b.logp_mu,
                                              b.adv, b.mask, **b.thresholds())
-        assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+        # the automatic shape keeps 128 KB of each row in tensor memory; a shape option the plain kernel
+        assert occ.occ_last_kernel() == ("k2_loss_l2/peel/tmem" if unroll is None else "k2_loss_l2/peel")
     torch.cuda.synchronize()
     s = occ.decode_loss_stats(out["stats"])
     near = np.minimum(o["dist_rd"], o["dist_rs"]) <= 1e-6

@@ -218,6 +218,8 @@ def test_misaligned_rows_with_matching_gradient_layout(dtype, V):
     the last row in its scalar tail."""
     T, off = 29, 1
     b, lp_old64 = _edge_batch(T, V, dtype, seed=V + 1, ld=V + 1, offset=off)
+    peeled = expected_kernel("k2", V, b.z_theta.element_size())  # "/tmem": the f32 rows
+    assert peeled.startswith("k2_loss_l2/peel")
     stride = b.z_theta.stride(0)
     assert stride % 2 == 1 and b.z_theta.data_ptr() % 16 != 0
     lp_th64, lse = logprob_rows(b.z_theta, b.ids, np.arange(T))
@@ -225,7 +227,7 @@ def test_misaligned_rows_with_matching_gradient_layout(dtype, V):
     dz_buf = torch.full((T, stride), 7.0, dtype=dtype, device="cuda")
     dz = dz_buf[:, off:off + V]
     out = _run(b, fp32(lp_old64), dz=dz)
-    assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    assert occ.occ_last_kernel() == peeled
     out["dlogits"] = dz
     _compare(b, out, o, lp_th64, dz_rows=np.arange(T), lse=lse, out_f32=dtype == torch.float32)
     assert torch.all(dz_buf[:, :off] == 7.0) and torch.all(dz_buf[:, off + V:] == 7.0)
@@ -236,10 +238,10 @@ def test_misaligned_rows_with_matching_gradient_layout(dtype, V):
     lp_old = torch.from_numpy(fp32(lp_old64)).to("cuda")
     out2 = occ.occ_decoupled_loss_fwd_bwd(z2, b.ids, lp_old, b.logp_mu, b.adv, b.mask,
                                           dlogits="inplace", **b.thresholds())
-    assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    assert occ.occ_last_kernel() == peeled
     # forward only
     out3 = _run(b, fp32(lp_old64), dz=None)
-    assert occ.occ_last_kernel() == "k2_loss_l2/peel"
+    assert occ.occ_last_kernel() == peeled
     assert torch.equal(z2, dz) and torch.equal(out2["stats"], out["stats"])
     assert torch.equal(out3["stats"], out["stats"]) and torch.equal(out3["logp"], out["logp"])
 

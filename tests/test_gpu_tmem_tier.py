@@ -178,3 +178,19 @@ def test_short_row_tier_equals_plain_kernels(V, T):
     assert ktm == expected_kernel("k2", V, es) and kpl == "k2_loss_l2"
     assert ktm == ("k2_loss_l2" if V == 24000 else "k2_loss_l2/tmem")
     _same(tm, pl)
+
+
+@pytest.mark.parametrize("V", [151937, 50257, 32001])
+def test_peeled_rows_tier_equals_plain_kernels(V):
+    # rows with an odd stride start at every residue modulo 16 bytes: the peeled
+    # kernels, in the 512-, 256- and 128-thread tiers
+    b = make_loss_batch("agentic_bf16_v151936", T=40, V=V, seed=V, device="cuda")
+    assert b.z_theta.stride(0) % 2 == 1
+    (tm, ktm), (pl, kpl) = _both(b)
+    assert ktm == expected_kernel("fused", V, 2, diag=False) == "k2_fused_l2/peel/tmem"
+    assert kpl == "k2_fused_l2/peel"
+    _same(tm, pl)
+    lp_old, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    (tm, ktm), (pl, kpl) = _k2_both(b, lp_old)
+    assert ktm == expected_kernel("k2", V, 2) == "k2_loss_l2/peel/tmem" and kpl == "k2_loss_l2/peel"
+    _same(tm, pl)
