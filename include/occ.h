@@ -398,13 +398,13 @@ const char* occ_last_error(void);
 /* The row kernel that the last call on this host thread launched, as a static
  * string: "k1_logprob_warp", "k1_logprob_warp/peel", "k1_logprob_vec",
  * "k1_logprob_vec/peel", "k1_logprob_scalar",
- * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_l2/tmem", "k2_loss_stream",
- * "k2_fused_l2", "k2_fused_l2/peel", "k2_fused_l2/tmem", "k2_fused_stream",
- * "k3_ewma_vec", "k3_ewma_scalar", "k3_ewma_bf16" ("" when the call launched
- * none, e.g. T = 0 or an invalid argument), and "k2_loss_l2/peel/tmem",
- * "k2_fused_l2/peel/tmem".  "/peel" marks the vector kernel run on rows that
- * start off a 16-byte boundary, "/tmem" its tensor-memory tier.  Never freed;
- * valid until the next call on the thread. */
+ * "k2_loss_l2", "k2_loss_l2/peel", "k2_loss_l2/tmem", "k2_loss_l2/peel/tmem",
+ * "k2_loss_stream", "k2_fused_l2", "k2_fused_l2/peel", "k2_fused_l2/tmem",
+ * "k2_fused_l2/peel/tmem", "k2_fused_stream", "k3_ewma_vec", "k3_ewma_scalar",
+ * "k3_ewma_bf16"; "" when the call launched none (e.g. T = 0 or an invalid
+ * argument).  "/peel" marks the vector kernel run on rows that start off a
+ * 16-byte boundary, "/tmem" its tensor-memory tier.  Never freed; valid until
+ * the next call on the thread. */
 const char* occ_last_kernel(void);
 
 /* OCC_VERSION of the built library. */
