@@ -321,12 +321,14 @@ static FusedKern fused_kernel(int nt) {
                      : k2_fused_l2<Tin, Tout, kFusedThreads, U, DIAG, PEEL>;
 }
 
-// The tensor-memory tier's instantiation for a CTA size (4 row pairs in flight).
-template <typename Tin, typename Tout, bool PEEL>
+// The tensor-memory tier's instantiation for a CTA size (the plain kernel's
+// row pairs in flight).
+template <typename Tin, typename Tout, bool DIAG, bool PEEL>
 static FusedKern tm_kernel(int nt) {
-  return nt == kTmThreads ? k2_fused_l2<Tin, Tout, kTmThreads, kFusedUnroll, false, PEEL, true>
-         : nt == 256      ? k2_fused_l2<Tin, Tout, 256, kFusedUnroll, false, PEEL, true>
-                          : k2_fused_l2<Tin, Tout, 128, kFusedUnroll, false, PEEL, true>;
+  constexpr int U = DIAG ? kFusedUnrollDiag : kFusedUnroll;
+  return nt == kTmThreads ? k2_fused_l2<Tin, Tout, kTmThreads, U, DIAG, PEEL, true>
+         : nt == 256      ? k2_fused_l2<Tin, Tout, 256, U, DIAG, PEEL, true>
+                          : k2_fused_l2<Tin, Tout, 128, U, DIAG, PEEL, true>;
 }
 
 // Rows off a 16-byte boundary run the vector kernel peeled when the old-logits
@@ -377,17 +379,18 @@ static occ_status launch_fused(FusedArgs f, bool vec, cudaStream_t s) {
     // the walk; OCC_OPT_FUSED_TMEM = 0 or a shape option (OCC_OPT_FUSED_THREADS,
     // OCC_OPT_FUSED_HEAD_BYTES) keeps the plain kernel.
     bool tm = false;
-    if constexpr (!DIAG) {
+    {
       // rows of a peeled call lose up to VEC - 1 elements to their scalar lead
+      constexpr int U = DIAG ? kFusedUnrollDiag : kFusedUnroll;
       const int hb = nt == kTmThreads ? kTmHeadBlocks : 0;
       const int64_t nvec_min = (f.a.V - (peel ? Elem<Tin>::kVec - 1 : 0)) / Elem<Tin>::kVec;
-      const int64_t full_blocks = nvec_min / ((int64_t)kFusedUnroll * nt) * kFusedUnroll;
+      const int64_t full_blocks = nvec_min / ((int64_t)U * nt) * U;
       if ((vec || peel) && (nt == kTmThreads || nt == 256 || nt == 128) &&
           option(OCC_OPT_FUSED_TMEM) != 0 && nt_opt < 0 && head_opt < 0 && T < step &&
           full_blocks >= hb + kTmBlocks) {
-        FusedKern kt = tm_kernel<Tin, Tout, false>(nt);
+        FusedKern kt = tm_kernel<Tin, Tout, DIAG, false>(nt);
         if constexpr (sizeof(Tin) == sizeof(Tout))
-          if (peel) kt = tm_kernel<Tin, Tout, true>(nt);
+          if (peel) kt = tm_kernel<Tin, Tout, DIAG, true>(nt);
         const size_t tm_head = (size_t)hb * nt * 16;
         if (tm_head == 0 || two_cta_smem_budget((const void*)kt) >= tm_head) {
           kern = kt;

@@ -102,15 +102,32 @@ def test_tmem_tier_threshold(V):
     _same(tm, pl)
 
 
-def test_diagnostics_and_head_option_keep_the_plain_kernel():
+def test_diagnostics_tier_equals_plain_kernel():
+    # the entropy / KL outputs: the same tier with 3 row pairs in flight
+    b = make_loss_batch("agentic_bf16_v151936", T=200, seed=2, device="cuda")
+    (tm, ktm), (pl, kpl) = _both(b, want_diagnostics=True)
+    assert ktm == "k2_fused_l2/tmem" and kpl == "k2_fused_l2"
+    _same(tm, pl)
+    assert torch.equal(_bits(tm["entropy"]), _bits(pl["entropy"]))
+    assert torch.equal(_bits(tm["kl"]), _bits(pl["kl"]))
+
+
+def test_shape_options_keep_the_plain_kernels():
     b = make_loss_batch("agentic_bf16_v151936", T=16, seed=2, device="cuda")
-    occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
-                                 want_diagnostics=True, **b.thresholds())
-    assert occ.occ_last_kernel() == "k2_fused_l2"
     with occ.options(fused_head_bytes=65536):
         occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
                                      **b.thresholds())
         assert occ.occ_last_kernel() == "k2_fused_l2"
+    with occ.options(fused_threads=512):
+        occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                     **b.thresholds())
+        assert occ.occ_last_kernel() == "k2_fused_l2"
+    lp_old, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    for opt in (dict(k2_threads=512), dict(k2_head_bytes=65536), dict(k2_unroll=8)):
+        with occ.options(**opt):
+            occ.occ_decoupled_loss_fwd_bwd(b.z_theta, b.ids, lp_old, b.logp_mu, b.adv, b.mask,
+                                           **b.thresholds())
+            assert occ.occ_last_kernel() == "k2_loss_l2", opt
     torch.cuda.synchronize()
 
 
