@@ -8,12 +8,13 @@
 // token is never read.  The backward pass is the K2 one (the current row's
 // head from shared memory, the rest re-read from L2).
 //
-// Long rows (the 512-thread tier) keep more of the current row on chip: a
-// shared-memory head and, after it, 128 KB in tensor memory, which no step of
-// this path needs for matrix work.  Only the rest of the row is re-read from L2,
-// and the re-reads that the gradient writes would push out of L2 are gone.  That
-// kernel is persistent (two CTAs per SM, rows fetched from a counter), so each
-// CTA allocates its tensor memory once.
+// Rows long enough for it keep more of the current row on chip: after the
+// shared-memory head, 16 blocks of NT vectors in tensor memory (128 KB at 512
+// threads, 64 KB at 256, 32 KB at 128), which no step of this path needs for
+// matrix work.  Only the rest of the row is re-read from L2, and the re-reads
+// that the gradient writes would push out of L2 are gone.  That kernel is
+// persistent (1024 / NT CTAs per SM, rows fetched from a counter), so each CTA
+// allocates its tensor memory once.
 //
 // Diagnostics (optional, no extra HBM bytes): the entropy of pi_theta,
 // H = lse - E_p[z], and KL(pi_old || pi_theta) = E_{p_old}[z_old - z] -

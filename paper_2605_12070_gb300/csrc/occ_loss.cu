@@ -14,8 +14,11 @@
 // the CTA reduction and the token's scalars, the backward pass turns the
 // shared-memory part and the L2 re-read of the rest into dlogits.  So HBM
 // sees the logits once and dlogits once: V * sizeof(T) read per valid token
-// plus V * sizeof(T_out) written per token (a dropped token is not read).  A
-// scalar-load two-pass kernel handles rows that cannot be vectorised.
+// plus V * sizeof(T_out) written per token (a dropped token is not read).
+// Rows long enough for it keep another part in tensor memory (the tier of
+// occ_common.cuh), which shrinks the re-read that the dirty dlogits lines in
+// L2 would otherwise push out.  A scalar-load two-pass kernel handles rows
+// that cannot be vectorised.
 //
 // K0 counts the valid tokens N before K2 runs (the token-mean denominator is
 // needed by every row's gradient).  A final one-CTA kernel reduces the
@@ -41,9 +44,10 @@ namespace occ {
 // waits in L2 by the longer of the two passes (newest-first lets the first
 // lines wait through both).  dlogits are written evict-first.
 //
-// TM (long aligned rows, 512 threads): the tensor-memory tier of
-// occ_common.cuh keeps 128 KB more of the row on chip, and the kernel runs
-// persistent, two CTAs per SM fetching rows from the workspace's counter.
+// TM: the tensor-memory tier of occ_common.cuh keeps 16 more blocks of NT
+// vectors of the row on chip (128 KB at 512 threads, 64 KB at 256, 32 KB at
+// 128), and the kernel runs persistent, 1024 / NT CTAs per SM fetching rows
+// from the workspace's counter.
 template <typename Tin, typename Tout, int NT, int U, bool PEEL, bool TM = false>
 __global__ void __launch_bounds__(NT, 1024 / NT) k2_loss_l2(const K2Args a) {
   static_assert(!TM || NT == kTmThreads || NT == 256 || NT == 128, "the tensor-memory tier");
