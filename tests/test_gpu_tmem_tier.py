@@ -211,3 +211,31 @@ def test_peeled_rows_tier_equals_plain_kernels(V):
     (tm, ktm), (pl, kpl) = _k2_both(b, lp_old)
     assert ktm == expected_kernel("k2", V, 2) == "k2_loss_l2/peel/tmem" and kpl == "k2_loss_l2/peel"
     _same(tm, pl)
+
+
+def test_tmem_kernels_on_two_streams_at_once():
+    # a fused and a K2 launch of the tier on two streams may share SMs: their CTAs'
+    # tensor memory (NT / 2 columns each) fits the SM whenever their registers do
+    b = make_loss_batch("agentic_bf16_v151936", T=1200, seed=21, device="cuda")
+    g = make_loss_batch("grpo_bf16_v32000", T=3000, seed=22, device="cuda")
+    lp_old, _ = occ.occ_token_logprob(g.z_old, g.ids)
+    torch.cuda.synchronize()
+    ref_f = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                         **b.thresholds())
+    ref_k = occ.occ_decoupled_loss_fwd_bwd(g.z_theta, g.ids, lp_old, g.logp_mu, g.adv, g.mask,
+                                           **g.thresholds())
+    torch.cuda.synchronize()
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    outs = []
+    for _ in range(3):
+        with torch.cuda.stream(s1):
+            f = occ.occ_decoupled_loss_fused(b.z_theta, b.z_old, b.ids, b.logp_mu, b.adv, b.mask,
+                                             **b.thresholds())
+        with torch.cuda.stream(s2):
+            k = occ.occ_decoupled_loss_fwd_bwd(g.z_theta, g.ids, lp_old, g.logp_mu, g.adv, g.mask,
+                                               **g.thresholds())
+        outs.append((f, k))
+    torch.cuda.synchronize()
+    for f, k in outs:
+        _same(f, ref_f)
+        _same(k, ref_k)
