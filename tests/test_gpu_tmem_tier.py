@@ -239,3 +239,20 @@ def test_tmem_kernels_on_two_streams_at_once():
     for f, k in outs:
         _same(f, ref_f)
         _same(k, ref_k)
+
+
+def test_tmem_tiers_with_every_token_masked():
+    # no row is read: the CTAs allocate, fetch rows, write zero gradients and free
+    b = make_loss_batch("agentic_bf16_v151936", T=64, seed=31, device="cuda")
+    b.mask.zero_()
+    (tm, ktm), (pl, kpl) = _both(b)
+    assert ktm == "k2_fused_l2/tmem"
+    _same(tm, pl)
+    assert torch.all(tm["dlogits"] == 0)
+    st = occ.decode_loss_stats(tm["stats"])
+    assert st.n_valid == 0 and st.loss == 0.0
+    lp_old, _ = occ.occ_token_logprob(b.z_old, b.ids)
+    (tm, ktm), (pl, kpl) = _k2_both(b, lp_old)
+    assert ktm == "k2_loss_l2/tmem"
+    _same(tm, pl)
+    assert torch.all(tm["dlogits"] == 0)
